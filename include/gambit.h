@@ -1,0 +1,234 @@
+/*
+ * gambit.h - C ABI of the GB300 (sm_103a) beam-decode library.
+ *
+ * The library implements the data-parallel hot path of thought-level beam
+ * search ("Gambit", Algorithm 1): one decode step over a population of
+ * reasoning beams that share forked KV-cache prefixes, the scorer probe at
+ * thought boundaries, and the tournament's prune/branch, which keeps the
+ * top-scoring beams and forks their block tables without copying KV.
+ *
+ * Conventions for every entry point
+ * ---------------------------------
+ * - Every function returns a gb_status; nothing throws across the ABI.
+ *   gb_last_error() gives a short static description of the last host-side
+ *   failure of a pool.
+ * - Device work is enqueued asynchronously on the caller's stream
+ *   (gb_stream_t is cudaStream_t; NULL means the legacy default stream).
+ *   Host-side argument checks fail synchronously with GB_ERR_INVALID /
+ *   GB_ERR_STATE / GB_ERR_UNSUPPORTED before anything is enqueued.
+ * - Errors found on the device (out of pages, a bad slot id, a bounded wait
+ *   that ran out) are recorded in a device status word: the first error
+ *   sticks.  gb_pool_status() synchronises the stream and reads it.  A
+ *   decode step whose page allocation failed does nothing: it changes no
+ *   pool state and its attention outputs are zero.
+ * - Ownership: the library never allocates device memory.  The caller
+ *   allocates the KV pool and the metadata buffer (sizes from
+ *   gb_pool_workspace_bytes), keeps them alive until gb_pool_destroy(), and
+ *   frees them afterwards.  The opaque gb_pool handle is a small host
+ *   struct owned by the library.
+ * - Pointers named *_dev are device pointers; all others are host pointers.
+ * - Slots: a pool has max_beams slots; a slot is active while it holds a
+ *   beam.  Arrays indexed by slot have max_beams entries.
+ * - GQA: query head h reads KV head h / (num_q_heads / num_kv_heads).
+ */
+#ifndef GAMBIT_H
+#define GAMBIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int gb_status;
+#define GB_OK 0
+#define GB_ERR_INVALID 1     /* bad argument or slot id */
+#define GB_ERR_OOM 2         /* no free page (or a block table is full) */
+#define GB_ERR_CUDA 3        /* a CUDA runtime call failed */
+#define GB_ERR_STATE 4       /* call out of order (e.g. layers of a step, release of an inactive slot) */
+#define GB_ERR_TIMEOUT 5     /* a bounded device-side wait ran out */
+#define GB_ERR_UNSUPPORTED 6 /* shape/dtype combination without a kernel */
+
+/* Element types. */
+#define GB_F32 0
+#define GB_BF16 1
+
+/* Decode path selection for gb_decode_attention(). */
+#define GB_PATH_AUTO 0      /* grouped tensor-core path where a shared segment is dense enough */
+#define GB_PATH_PER_BEAM 1  /* every beam reads its whole context itself */
+#define GB_PATH_GROUPED 2   /* like AUTO (kept for explicit requests) */
+
+typedef struct CUstream_st* gb_stream_t; /* identical to cudaStream_t */
+typedef struct gb_pool gb_pool;          /* opaque host handle */
+
+typedef struct {
+  int num_layers;          /* layers sharing one page id space (a page spans all layers) */
+  int num_q_heads;         /* Hq */
+  int num_kv_heads;        /* Hkv; Hq % Hkv == 0 */
+  int head_dim;            /* D: 128 for GB_BF16, 64 for GB_F32 */
+  int page_size;           /* P tokens per page: 16, 32 or 64 */
+  int kv_dtype;            /* GB_F32 or GB_BF16: K/V storage and the query dtype */
+  int64_t num_pages;       /* pages in the pool */
+  int max_beams;           /* slots = capacity C of the tournament, <= 1024 */
+  int max_pages_per_beam;  /* block-table width */
+  int group_min_beams;     /* grouped path only for segments shared by >= this many beams (0: default 16) */
+} gb_pool_config;
+
+/* Host-side copies of the pool state, for tests and debugging (any member may be NULL). */
+typedef struct {
+  int32_t* tables;     /* [max_beams][max_pages_per_beam]; entries past ceil(seq_len/P) unspecified */
+  int32_t* seq_len;    /* [max_beams] tokens in each slot's context (0 when inactive) */
+  int32_t* active;     /* [max_beams] 1 when the slot holds a beam */
+  int32_t* gen;        /* [max_beams] tokens generated since the beam's own creation */
+  int32_t* nsteps;     /* [max_beams] scored thought steps n */
+  float* mean;         /* [max_beams] running mean score s_bar */
+  uint32_t* lineage;   /* [max_beams] unique id of the beam now in the slot */
+  int32_t* refcnt;     /* [num_pages] active slots referencing each page */
+  uint32_t* free_bits; /* [ceil(num_pages/32)] bit p%32 of word p/32 set when page p is free */
+} gb_pool_state;
+
+/*
+ * Sizes of the two caller-allocated device buffers for a configuration.
+ * kv_bytes: the paged KV pool, laid out [layer][page][K|V][kv_head][P][D] in
+ * kv_dtype.  meta_bytes: block tables, refcounts, free bitmap, per-slot
+ * scores, decode plans and split-KV partials.  Either output may be NULL.
+ * Paged KV and block tables: Section 3.1 (branching "via prefix caching",
+ * pruning "frees their non-shared KV-cache blocks").
+ * Errors: GB_ERR_INVALID for an inconsistent config, GB_ERR_UNSUPPORTED for
+ * a (kv_dtype, head_dim, Hq/Hkv) without a kernel.
+ */
+gb_status gb_pool_workspace_bytes(const gb_pool_config* cfg, size_t* kv_bytes, size_t* meta_bytes);
+
+/*
+ * Create a pool over caller memory.  kv_dev and meta_dev must be 256-byte
+ * aligned and at least the sizes above.  The metadata is initialised on
+ * `stream` (every page free, every slot inactive); K/V contents are left as
+ * they are.  *out receives the handle.
+ */
+gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void* meta_dev,
+                       gb_stream_t stream, gb_pool** out);
+
+/* Free the host handle (not the caller's device buffers). */
+gb_status gb_pool_destroy(gb_pool* pool);
+
+/*
+ * Seed the C initial traces of Algorithm 1 ("S <- C initial traces from P"):
+ * slots 0..n_beams-1 become active, all sharing the prompt's pages
+ * (refcount n_beams each, lowest free page ids).  k_prompt_dev/v_prompt_dev:
+ * [num_layers][prompt_len][Hkv][D] in kv_dtype.  Running means start at 0
+ * with n = 0.  Slots get lineage ids in order.
+ * Errors: GB_ERR_STATE unless every slot is inactive; GB_ERR_INVALID for a
+ * bad count or length; out of pages is reported in the device status.
+ */
+gb_status gb_pool_seed(gb_pool* pool, int n_beams, int prompt_len, const void* k_prompt_dev,
+                       const void* v_prompt_dev, gb_stream_t stream);
+
+/*
+ * One decode step of one layer for every active beam (Algorithm 1,
+ * "Generate: advance one thought for all tau in S", one token at a time).
+ * Appends k_new/v_new at each beam's next position, then computes GQA decode
+ * attention over the beam's whole context through its block table:
+ *   out[b][h] = sum_t softmax_t(scale * q[b][h] . K_b[t]) V_b[t]
+ * where K_b/V_b are read from KV head h / G.  Layer 0 opens a step (reserves
+ * the position for every beam, allocating the lowest free page at a page
+ * boundary and copying a still-shared partial tail page); layers must then be
+ * called in order 0..num_layers-1.
+ *   q_dev:      [max_beams][Hq][D] in kv_dtype
+ *   k_new_dev, v_new_dev: [max_beams][Hkv][D] in kv_dtype
+ *   out_dev:    [max_beams][Hq][D] fp32 (rows of inactive slots are zero)
+ *   flags:      GB_PATH_AUTO / GB_PATH_PER_BEAM / GB_PATH_GROUPED
+ * Rows of inactive slots in the inputs are ignored.
+ * Errors: GB_ERR_STATE for a layer out of order; out of pages is reported in
+ * the device status and makes the whole step a no-op.
+ */
+gb_status gb_decode_attention(gb_pool* pool, int layer, const void* q_dev, const void* k_new_dev,
+                              const void* v_new_dev, float scale, float* out_dev, int flags,
+                              gb_stream_t stream);
+
+/*
+ * Append n_tokens tokens to every active beam for one layer, without
+ * attention (a chunk of a thought written at once).  Equivalent to n_tokens
+ * decode steps' appends: page allocation follows the same order (token by
+ * token, slots ascending).  k_dev/v_dev: [n_tokens][max_beams][Hkv][D].
+ * Layer 0 reserves the positions; layers 1.. must follow in order.
+ * Errors as gb_decode_attention.
+ */
+gb_status gb_append_kv(gb_pool* pool, int layer, int n_tokens, const void* k_dev,
+                       const void* v_dev, gb_stream_t stream);
+
+/*
+ * Scorer probe at a thought boundary and the running-mean update of
+ * Algorithm 1 ("s_bar <- s_bar + (f(h_n) - s_bar)/n"), with the probe
+ * f(h) = sigmoid(w . h + bias) (Section 3.1 scores traces with a light-weight
+ * scorer on the last-layer hidden state).
+ *   hidden_dev:  [max_beams][hidden_dim] in hidden_dtype (GB_F32/GB_BF16)
+ *   w_dev:       [hidden_dim] fp32
+ *   boundary_mask_dev: [max_beams] u8, or NULL for every active slot; only
+ *                masked active slots update (n += 1, s_bar updated in fp32:
+ *                subtract, divide, add, each rounded)
+ *   score_out_dev: [max_beams] fp32 probe score (0 for inactive slots), may be NULL
+ * Errors: GB_ERR_INVALID unless hidden_dim is a positive multiple of 8.
+ */
+gb_status gb_score_probe(gb_pool* pool, const void* hidden_dev, int hidden_dtype, int hidden_dim,
+                         const float* w_dev, float bias, const uint8_t* boundary_mask_dev,
+                         float* score_out_dev, gb_stream_t stream);
+
+/*
+ * Running-mean update with scores computed elsewhere (any scorer f_theta,
+ * Section 3.1): for masked active slots, n += 1 and s_bar is updated exactly
+ * as in gb_score_probe.  scores_dev: [max_beams] fp32; mask as above.
+ */
+gb_status gb_push_scores(gb_pool* pool, const float* scores_dev, const uint8_t* mask_dev,
+                         gb_stream_t stream);
+
+/*
+ * One tournament round (Algorithm 1, Tournament; Eq. 2 and Eq. 3).
+ * Active slots are ranked by s_bar descending (ties: lower slot first; NaN
+ * last).  Eligible parents are active slots with gen >= warmup and, when
+ * eligible_dev is given, eligible_dev[slot] != 0.
+ *   Case 1 (fewer active slots than max_beams): the top min(vacant, |B|)
+ *   eligible beams get one child each, placed in vacant slots ascending.
+ *   Case 2 (all slots active): prune the bottom K_eff = min(K, (fanout-1) x
+ *   eligible survivors) beams; each of the top eligible survivors gets
+ *   fanout-1 children (the last one the remainder), placed in the pruned
+ *   slots ascending.  fanout = 2 is Eq. 3 exactly.
+ * A child gets its parent's block table (every page's refcount + 1; no KV is
+ * copied), length, s_bar and n, gen = 0 and a new lineage id.  A pruned beam
+ * drops its references; pages reaching refcount 0 become free.
+ *   parent_out_dev:  [max_beams] int32: own slot for surviving beams, parent
+ *                    slot for new children, -1 for inactive slots (may be NULL)
+ *   pruned_out_dev:  [max_beams] u8: 1 where a beam was pruned (may be NULL)
+ *   lineage_out_dev: [max_beams] u32 lineage ids after the round (may be NULL)
+ * Errors: GB_ERR_INVALID for K < 0 or fanout < 2.
+ */
+gb_status gb_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const uint8_t* eligible_dev,
+                          int32_t* parent_out_dev, uint8_t* pruned_out_dev, uint32_t* lineage_out_dev,
+                          gb_stream_t stream);
+
+/*
+ * Release slots whose traces completed ("move completed traces to F") or
+ * were evicted as ghost traces (Section 3.2): each listed slot drops its page
+ * references (pages reaching 0 become free) and becomes inactive.  slots_dev:
+ * [n] int32 device array, processed in order.  A slot out of range records
+ * GB_ERR_INVALID, an inactive slot GB_ERR_STATE, in the device status; the
+ * entry is skipped.
+ */
+gb_status gb_release(gb_pool* pool, const int32_t* slots_dev, int n, gb_stream_t stream);
+
+/* Synchronise `stream` and read the device status word (GB_OK or the first error). */
+gb_status gb_pool_status(gb_pool* pool, int* device_status, gb_stream_t stream);
+
+/* Reset the device status word to GB_OK (enqueued on `stream`). */
+gb_status gb_pool_clear_status(gb_pool* pool, gb_stream_t stream);
+
+/* Synchronise `stream` and copy the pool state into host arrays (see gb_pool_state). */
+gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_stream_t stream);
+
+/* Short description of the pool's last host-side failure ("" if none); static storage. */
+const char* gb_last_error(gb_pool* pool);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GAMBIT_H */

@@ -1,0 +1,189 @@
+"""ctypes binding of ``libgambit.so`` (the C ABI declared in ``include/gambit.h``).
+
+Argument marshalling only: every step of the hot path runs in the library's
+CUDA kernels.  Device arguments may be torch tensors (their ``data_ptr()`` is
+passed) or raw integer device addresses; streams may be ``torch.cuda.Stream``
+objects, raw ``cudaStream_t`` integers or ``None`` (the current torch stream
+when torch is initialised on CUDA, else the legacy default stream).
+
+If the shared library has not been built the import of this module succeeds
+but the first call raises ``RuntimeError``: there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+
+LIB_PATH = Path(__file__).resolve().with_name("libgambit.so")
+
+GB_OK, GB_ERR_INVALID, GB_ERR_OOM, GB_ERR_CUDA, GB_ERR_STATE, GB_ERR_TIMEOUT, GB_ERR_UNSUPPORTED = range(7)
+STATUS_NAMES = {0: "GB_OK", 1: "GB_ERR_INVALID", 2: "GB_ERR_OOM", 3: "GB_ERR_CUDA", 4: "GB_ERR_STATE",
+                5: "GB_ERR_TIMEOUT", 6: "GB_ERR_UNSUPPORTED"}
+GB_F32, GB_BF16 = 0, 1
+GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
+
+# Every symbol the header declares, in header order.
+EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
+           "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
+           "gb_pool_clear_status", "gb_pool_read_state", "gb_last_error"]
+
+
+class GbPoolConfig(ctypes.Structure):
+    _fields_ = [("num_layers", ctypes.c_int), ("num_q_heads", ctypes.c_int), ("num_kv_heads", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("page_size", ctypes.c_int), ("kv_dtype", ctypes.c_int),
+                ("num_pages", ctypes.c_int64), ("max_beams", ctypes.c_int), ("max_pages_per_beam", ctypes.c_int),
+                ("group_min_beams", ctypes.c_int)]
+
+
+class GbPoolState(ctypes.Structure):
+    _fields_ = [("tables", ctypes.c_void_p), ("seq_len", ctypes.c_void_p), ("active", ctypes.c_void_p),
+                ("gen", ctypes.c_void_p), ("nsteps", ctypes.c_void_p), ("mean", ctypes.c_void_p),
+                ("lineage", ctypes.c_void_p), ("refcnt", ctypes.c_void_p), ("free_bits", ctypes.c_void_p)]
+
+
+class GambitError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        super().__init__(f"{STATUS_NAMES.get(code, code)}: {what}")
+        self.code = code
+
+
+_lib = None
+
+
+def load(path: Path | None = None) -> ctypes.CDLL:
+    """Load the library (once).  Raises RuntimeError when it has not been built."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = Path(path) if path else LIB_PATH
+    if not p.exists():
+        raise RuntimeError(f"{p} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(str(p))
+    V, I, F, P = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_void_p
+    sig = {
+        "gb_pool_workspace_bytes": [P, P, P],
+        "gb_pool_init": [P, V, V, V, P],
+        "gb_pool_destroy": [V],
+        "gb_pool_seed": [V, I, I, V, V, V],
+        "gb_decode_attention": [V, I, V, V, V, F, V, I, V],
+        "gb_append_kv": [V, I, I, V, V, V],
+        "gb_score_probe": [V, V, I, I, V, F, V, V, V],
+        "gb_push_scores": [V, V, V, V],
+        "gb_prune_branch": [V, I, I, I, V, V, V, V, V],
+        "gb_release": [V, V, I, V],
+        "gb_pool_status": [V, P, V],
+        "gb_pool_clear_status": [V, V],
+        "gb_pool_read_state": [V, P, V],
+        "gb_last_error": [V],
+    }
+    for name, args in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = ctypes.c_char_p if name == "gb_last_error" else ctypes.c_int
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def ptr(x) -> int | None:
+    """Device address of a tensor / int, or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def stream_handle(s) -> int | None:
+    if s is None:
+        try:
+            import torch
+            if torch.cuda.is_available() and torch.cuda.is_initialized():
+                return torch.cuda.current_stream().cuda_stream
+        except Exception:
+            pass
+        return None
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def _check(pool_handle, code: int, what: str) -> None:
+    if code != GB_OK:
+        detail = load().gb_last_error(pool_handle) if pool_handle else b""
+        raise GambitError(code, f"{what}: {(detail or b'').decode()}")
+
+
+# ---------------------------------------------------------------------------
+# Functions with the C names (raise GambitError on a non-OK status).
+# ---------------------------------------------------------------------------
+
+def gb_pool_workspace_bytes(cfg: GbPoolConfig) -> tuple[int, int]:
+    kv, meta = ctypes.c_size_t(), ctypes.c_size_t()
+    _check(None, load().gb_pool_workspace_bytes(ctypes.byref(cfg), ctypes.byref(kv), ctypes.byref(meta)),
+           "gb_pool_workspace_bytes")
+    return kv.value, meta.value
+
+
+def gb_pool_init(cfg: GbPoolConfig, kv_dev, meta_dev, stream=None) -> int:
+    h = ctypes.c_void_p()
+    _check(None, load().gb_pool_init(ctypes.byref(cfg), ptr(kv_dev), ptr(meta_dev), stream_handle(stream),
+                                     ctypes.byref(h)), "gb_pool_init")
+    return h.value
+
+
+def gb_pool_destroy(pool: int) -> None:
+    load().gb_pool_destroy(pool)
+
+
+def gb_pool_seed(pool: int, n_beams: int, prompt_len: int, k_prompt, v_prompt, stream=None) -> None:
+    _check(pool, load().gb_pool_seed(pool, n_beams, prompt_len, ptr(k_prompt), ptr(v_prompt),
+                                     stream_handle(stream)), "gb_pool_seed")
+
+
+def gb_decode_attention(pool: int, layer: int, q, k_new, v_new, scale: float, out, flags: int = GB_PATH_AUTO,
+                        stream=None) -> None:
+    _check(pool, load().gb_decode_attention(pool, layer, ptr(q), ptr(k_new), ptr(v_new), float(scale), ptr(out),
+                                            flags, stream_handle(stream)), "gb_decode_attention")
+
+
+def gb_append_kv(pool: int, layer: int, n_tokens: int, k, v, stream=None) -> None:
+    _check(pool, load().gb_append_kv(pool, layer, n_tokens, ptr(k), ptr(v), stream_handle(stream)), "gb_append_kv")
+
+
+def gb_score_probe(pool: int, hidden, hidden_dtype: int, hidden_dim: int, w, bias: float, mask=None,
+                   score_out=None, stream=None) -> None:
+    _check(pool, load().gb_score_probe(pool, ptr(hidden), hidden_dtype, hidden_dim, ptr(w), float(bias), ptr(mask),
+                                       ptr(score_out), stream_handle(stream)), "gb_score_probe")
+
+
+def gb_push_scores(pool: int, scores, mask=None, stream=None) -> None:
+    _check(pool, load().gb_push_scores(pool, ptr(scores), ptr(mask), stream_handle(stream)), "gb_push_scores")
+
+
+def gb_prune_branch(pool: int, K: int, fanout: int, warmup: int = 0, eligible=None, parent_out=None,
+                    pruned_out=None, lineage_out=None, stream=None) -> None:
+    _check(pool, load().gb_prune_branch(pool, K, fanout, warmup, ptr(eligible), ptr(parent_out), ptr(pruned_out),
+                                        ptr(lineage_out), stream_handle(stream)), "gb_prune_branch")
+
+
+def gb_release(pool: int, slots, n: int, stream=None) -> None:
+    _check(pool, load().gb_release(pool, ptr(slots), n, stream_handle(stream)), "gb_release")
+
+
+def gb_pool_status(pool: int, stream=None) -> int:
+    st = ctypes.c_int()
+    _check(pool, load().gb_pool_status(pool, ctypes.byref(st), stream_handle(stream)), "gb_pool_status")
+    return st.value
+
+
+def gb_pool_clear_status(pool: int, stream=None) -> None:
+    _check(pool, load().gb_pool_clear_status(pool, stream_handle(stream)), "gb_pool_clear_status")
+
+
+def gb_pool_read_state(pool: int, state: GbPoolState, stream=None) -> None:
+    _check(pool, load().gb_pool_read_state(pool, ctypes.byref(state), stream_handle(stream)), "gb_pool_read_state")
+
+
+def gb_last_error(pool: int) -> str:
+    return (load().gb_last_error(pool) or b"").decode()

@@ -1,0 +1,471 @@
+// Split-KV flash-decode over the paged pool (per-beam path) and the LSE combine.
+//
+// Work decomposition: the per-beam work of a step is the flat list of
+// (beam, kv-head, 16-token chunk) units, ordered beam-major.  Every warp of a
+// persistent grid takes one contiguous range of that list, so work is
+// balanced to within one chunk whatever the beams' lengths.  A warp streams
+// its chunks through a private ring of shared-memory stages filled by 1D
+// bulk copies (TMA): one 4 KiB K slab and one 4 KiB V slab per chunk, both
+// contiguous in a page.  When its range leaves a (beam, head) it writes an
+// unnormalised partial (m, l, o) for the G query heads of that KV head; the
+// combine kernel merges the partials of each (beam, head) with the standard
+// log-sum-exp rule.
+//
+// Lane layout inside a warp: 4 token rows x 8 lanes.  Lane j of row r owns
+// two 16-byte pieces of every token row (bytes [16j, 16j+16) and
+// [128+16j, 128+16j+16) of the 256-byte row), i.e. 16 bf16 or 8 fp32 dims,
+// and handles tokens r, r+4, r+8, r+12 of a chunk.  Scores are reduced with
+// a 3-stage shuffle reduce-scatter inside each 8-lane row; softmax maxima
+// are warp-wide so rescaling is a warp-uniform branch.
+#include <math.h>
+
+#include "internal.cuh"
+#include "ptx.cuh"
+
+namespace gb {
+
+template <int DT>
+struct KvTraits {
+  static constexpr int ES = DT == GB_BF16 ? 2 : 4;
+  static constexpr int D = DT == GB_BF16 ? 128 : 64;
+  static constexpr int DPC = 16 / ES;  // dims per 16-byte piece
+  static constexpr int DPL = 2 * DPC;  // dims per lane
+  static constexpr int ROW_BYTES = D * ES;
+  static constexpr int SLAB_BYTES = kChunk * ROW_BYTES;  // 4096
+  static constexpr int STAGE_BYTES = 2 * SLAB_BYTES;     // K + V
+  static_assert(ROW_BYTES == 256, "lane layout assumes 256-byte token rows");
+};
+
+// Unpack one 16-byte piece into DPC floats.
+template <int DT>
+__device__ __forceinline__ void unpack16(const uint4& u, float* f) {
+  if constexpr (DT == GB_BF16) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      f[2 * k] = __uint_as_float(w[k] << 16);
+      f[2 * k + 1] = __uint_as_float(w[k] & 0xffff0000u);
+    }
+  } else {
+    f[0] = __uint_as_float(u.x);
+    f[1] = __uint_as_float(u.y);
+    f[2] = __uint_as_float(u.z);
+    f[3] = __uint_as_float(u.w);
+  }
+}
+
+template <int DT, int G>
+struct DecodeSmem {
+  using T = KvTraits<DT>;
+  static constexpr int PBUF = kChunk * G * 4;
+  // Rounded to 128 bytes so every warp's stages start 16-byte aligned (bulk-copy destinations).
+  static constexpr int WARP_BYTES = (kDecodeStages * T::STAGE_BYTES + PBUF + 8 * kDecodeStages + 127) / 128 * 128;
+  static_assert(WARP_BYTES % 128 == 0 && T::STAGE_BYTES % 16 == 0, "stage alignment");
+  static constexpr int PLAN_BYTES = 3 * (kMaxBeams + 1) * 4;
+  static constexpr int TOTAL = kDecodeWarps * WARP_BYTES + PLAN_BYTES;
+};
+
+struct ChunkIter {
+  int b, h, i, n, tok0;
+};
+
+__device__ __forceinline__ void iter_advance(ChunkIter& it, const int* s_n, const int* s_start, int Hkv,
+                                             int max_beams) {
+  if (++it.i == it.n) {
+    it.i = 0;
+    if (++it.h == Hkv) {
+      it.h = 0;
+      do {
+        ++it.b;
+      } while (it.b < max_beams && s_n[it.b] == 0);
+      if (it.b < max_beams) {
+        it.n = s_n[it.b];
+        it.tok0 = s_start[it.b];
+      }
+    }
+  }
+}
+
+template <int DT, int G>
+__global__ void __launch_bounds__(kDecodeWarps * 32, 1)
+    k_decode(PoolView v, int layer, const void* __restrict__ qptr, float qscale, int mode, int W) {
+  using T = KvTraits<DT>;
+  using S = DecodeSmem<DT, G>;
+  constexpr int NS = G / 2;  // scores held per lane after the reduce-scatter
+  constexpr int D = T::D, DPC = T::DPC, DPL = T::DPL;
+  extern __shared__ __align__(128) unsigned char smem[];
+
+  int* s_off = reinterpret_cast<int*>(smem + kDecodeWarps * S::WARP_BYTES);
+  int* s_n = s_off + (kMaxBeams + 1);
+  int* s_start = s_n + (kMaxBeams + 1);
+  if (v.ctl[kCtlStepOk] == 0) return;
+  {
+    const int* off = plan_off(v, mode);
+    const int* nn = plan_n(v, mode);
+    const int* st = plan_start(v, mode);
+    for (int i = threadIdx.x; i <= v.max_beams; i += blockDim.x) {
+      s_off[i] = off[i];
+      s_n[i] = i < v.max_beams ? nn[i] : 0;
+      s_start[i] = i < v.max_beams ? st[i] : 0;
+    }
+  }
+  __syncthreads();
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = lane >> 3, j = lane & 7;
+  const int b0 = lane & 1, b1 = (lane >> 1) & 1, b2 = (lane >> 2) & 1;
+  const int my_t = 4 * (2 * b2 + b1) + row;  // token (within the chunk) of this lane's scores
+  unsigned char* wsm = smem + warp * S::WARP_BYTES;
+  float* pbuf = reinterpret_cast<float*>(wsm + kDecodeStages * T::STAGE_BYTES);
+  const uint32_t stage0 = smem_addr(wsm);
+  const uint32_t bar0 = smem_addr(wsm + kDecodeStages * T::STAGE_BYTES + S::PBUF);
+
+  const int Tot = s_off[v.max_beams];
+  const int w = blockIdx.x * kDecodeWarps + warp;
+  const int c = (Tot + W - 1) / W;
+  const int x_begin = w * c;
+  const int x_end = min(Tot, x_begin + c);
+  if (x_begin >= x_end) return;
+
+  if (lane == 0) {
+    for (int s = 0; s < kDecodeStages; ++s) mbar_init(bar0 + 8 * s, 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+
+  // Locate the first chunk: the largest b with s_off[b] <= x_begin.
+  ChunkIter it;
+  {
+    int lo = 0, hi = v.max_beams;  // invariant: s_off[lo] <= x < s_off[hi]
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      if (s_off[mid] <= x_begin) lo = mid; else hi = mid;
+    }
+    it.b = lo;
+    it.n = s_n[lo];
+    it.tok0 = s_start[lo];
+    const int r = x_begin - s_off[lo];
+    it.h = r / it.n;
+    it.i = r % it.n;
+  }
+  const uint64_t pol = policy_evict_first();
+  auto load_page = [&](const ChunkIter& q) -> int {
+    const int tok = q.tok0 + q.i * kChunk;
+    int page = v.tables[(size_t)q.b * v.max_pages + tok / v.P];
+    return page;
+  };
+  auto issue = [&](const ChunkIter& q, int page, int stage) {
+    if (lane == 0) {
+      if (page < 0 || page >= v.num_pages) {
+        set_status(v.ctl, GB_ERR_INVALID);
+        page = 0;
+      }
+      const int tok = q.tok0 + q.i * kChunk;
+      const long long ek = kv_elem_offset(v, layer, page, 0, q.h, tok % v.P);
+      const long long ev = kv_elem_offset(v, layer, page, 1, q.h, tok % v.P);
+      const uint32_t bar = bar0 + 8 * stage;
+      const uint32_t dst = stage0 + stage * T::STAGE_BYTES;
+      mbar_arrive_expect_tx(bar, T::STAGE_BYTES);
+      bulk_g2s(dst, v.kv + ek * T::ES, T::SLAB_BYTES, bar, pol);
+      bulk_g2s(dst + T::SLAB_BYTES, v.kv + ev * T::ES, T::SLAB_BYTES, bar, pol);
+    }
+  };
+
+  // Prologue: fill the ring.
+  ChunkIter ip = it;
+  int ip_x = x_begin;
+  int ip_page = load_page(ip);
+  for (int s = 0; s < kDecodeStages; ++s) {
+    if (ip_x < x_end) {
+      issue(ip, ip_page, s);
+      ++ip_x;
+      if (ip_x < x_end) {
+        iter_advance(ip, s_n, s_start, v.Hkv, v.max_beams);
+        ip_page = load_page(ip);
+      }
+    }
+  }
+
+  float qr[G][DPL];
+  float o[G][DPL];
+  float m_run[G];
+  float l_lane[NS];
+  int L = 0;
+  bool fresh = true;
+  const char* qbase = static_cast<const char*>(qptr);
+
+  for (int x = x_begin, k = 0; x < x_end; ++x, ++k) {
+    if (fresh) {
+      // New (beam, head): load the G query rows for this lane's dims, pre-scaled.
+      L = v.seq_len[it.b];
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const char* qrow = qbase + ((size_t)(it.b * v.Hq + it.h * G + g) * D) * T::ES;
+        const uint4 a = *reinterpret_cast<const uint4*>(qrow + 16 * j);
+        const uint4 bq = *reinterpret_cast<const uint4*>(qrow + 128 + 16 * j);
+        unpack16<DT>(a, qr[g]);
+        unpack16<DT>(bq, qr[g] + DPC);
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) {
+          qr[g][d] *= qscale;
+          o[g][d] = 0.f;
+        }
+        m_run[g] = -INFINITY;
+      }
+#pragma unroll
+      for (int kk = 0; kk < NS; ++kk) l_lane[kk] = 0.f;
+      fresh = false;
+    }
+    const int stage = k % kDecodeStages;
+    const uint32_t parity = (k / kDecodeStages) & 1;
+    if (!mbar_wait_bounded(bar0 + 8 * stage, parity, kWaitLimitNs)) {
+      if (lane == 0) set_status(v.ctl, GB_ERR_TIMEOUT);
+      // Give copies still in flight a bounded chance to land before leaving.
+      for (int s = 0; s < kDecodeStages; ++s) {
+        const int kk = k + s;
+        if (x + s < ip_x) mbar_wait_bounded(bar0 + 8 * (kk % kDecodeStages), (kk / kDecodeStages) & 1, kWaitLimitNs / 4);
+      }
+      return;
+    }
+    const unsigned char* Ks = wsm + stage * T::STAGE_BYTES;
+    const unsigned char* Vs = Ks + T::SLAB_BYTES;
+    const int tok0 = it.tok0 + it.i * kChunk;
+    const bool partial = tok0 + kChunk > L;
+
+    // ---- scores: 4 tokens per row, G heads each --------------------------
+    float acc[4 * G];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int t = 4 * i + row;
+      const uint4 a = *reinterpret_cast<const uint4*>(Ks + t * T::ROW_BYTES + 16 * j);
+      const uint4 bq = *reinterpret_cast<const uint4*>(Ks + t * T::ROW_BYTES + 128 + 16 * j);
+      float kf[DPL];
+      unpack16<DT>(a, kf);
+      unpack16<DT>(bq, kf + DPC);
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        float sacc = 0.f;
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) sacc = fmaf(qr[g][d], kf[d], sacc);
+        acc[i * G + g] = sacc;
+      }
+    }
+    // Reduce-scatter over the 8 lanes of the row: 4G -> 2G -> G -> G/2 values.
+#pragma unroll
+    for (int kk = 0; kk < 2 * G; ++kk) {
+      const bool up = lane & 4;
+      const float keep = up ? acc[kk + 2 * G] : acc[kk];
+      const float send = up ? acc[kk] : acc[kk + 2 * G];
+      acc[kk] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+    }
+#pragma unroll
+    for (int kk = 0; kk < G; ++kk) {
+      const bool up = lane & 2;
+      const float keep = up ? acc[kk + G] : acc[kk];
+      const float send = up ? acc[kk] : acc[kk + G];
+      acc[kk] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+    }
+    float sc[NS];
+#pragma unroll
+    for (int kk = 0; kk < NS; ++kk) {
+      const bool up = lane & 1;
+      const float keep = up ? acc[kk + NS] : acc[kk];
+      const float send = up ? acc[kk] : acc[kk + NS];
+      sc[kk] = keep + __shfl_xor_sync(0xffffffffu, send, 1);
+      if (partial && tok0 + my_t >= L) sc[kk] = -INFINITY;
+    }
+    // ---- online softmax (warp-wide maxima, base 2) -------------------------
+    float mx[NS], other[NS];
+#pragma unroll
+    for (int kk = 0; kk < NS; ++kk) {
+      float m = sc[kk];
+      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
+      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 4));
+      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 8));
+      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 16));
+      mx[kk] = m;
+    }
+#pragma unroll
+    for (int kk = 0; kk < NS; ++kk) other[kk] = __shfl_xor_sync(0xffffffffu, mx[kk], 1);
+    bool grow = false;
+    float m_new[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const float mc = ((g / NS) == b0) ? mx[g % NS] : other[g % NS];
+      m_new[g] = fmaxf(m_run[g], mc);
+      grow |= m_new[g] > m_run[g];
+    }
+    if (grow) {
+      float alpha[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        alpha[g] = exp2f(m_run[g] - m_new[g]);
+        m_run[g] = m_new[g];
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) o[g][d] *= alpha[g];
+      }
+#pragma unroll
+      for (int kk = 0; kk < NS; ++kk) l_lane[kk] *= b0 ? alpha[NS + kk] : alpha[kk];
+    }
+#pragma unroll
+    for (int kk = 0; kk < NS; ++kk) {
+      const float mr = b0 ? m_run[NS + kk] : m_run[kk];
+      const float p = exp2f(sc[kk] - mr);
+      l_lane[kk] += p;
+      pbuf[my_t * G + NS * b0 + kk] = p;
+    }
+    __syncwarp();
+    // ---- P.V -----------------------------------------------------------------
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int t = 4 * i + row;
+      float pv[G];
+#pragma unroll
+      for (int g = 0; g < G; ++g) pv[g] = pbuf[t * G + g];
+      const uint4 a = *reinterpret_cast<const uint4*>(Vs + t * T::ROW_BYTES + 16 * j);
+      const uint4 bq = *reinterpret_cast<const uint4*>(Vs + t * T::ROW_BYTES + 128 + 16 * j);
+      float vf[DPL];
+      unpack16<DT>(a, vf);
+      unpack16<DT>(bq, vf + DPC);
+      if (partial && tok0 + t >= L) {
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) vf[d] = 0.f;
+      }
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) o[g][d] = fmaf(pv[g], vf[d], o[g][d]);
+    }
+    __syncwarp();
+    // The stage is free again: refill it with the chunk kDecodeStages ahead.
+    if (ip_x < x_end) {
+      if (lane == 0) fence_proxy_async_smem();
+      issue(ip, ip_page, stage);
+      ++ip_x;
+      if (ip_x < x_end) {
+        iter_advance(ip, s_n, s_start, v.Hkv, v.max_beams);
+        ip_page = load_page(ip);
+      }
+    }
+    // ---- end of this warp's share of (beam, head): write the partial --------
+    const bool last_of_bh = (it.i == it.n - 1) || (x + 1 == x_end);
+    if (last_of_bh) {
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int d = 0; d < DPL; ++d) {
+          o[g][d] += __shfl_xor_sync(0xffffffffu, o[g][d], 8);
+          o[g][d] += __shfl_xor_sync(0xffffffffu, o[g][d], 16);
+        }
+      float lsum[NS], lother[NS];
+#pragma unroll
+      for (int kk = 0; kk < NS; ++kk) {
+        float s = l_lane[kk];
+        s += __shfl_xor_sync(0xffffffffu, s, 2);
+        s += __shfl_xor_sync(0xffffffffu, s, 4);
+        s += __shfl_xor_sync(0xffffffffu, s, 8);
+        s += __shfl_xor_sync(0xffffffffu, s, 16);
+        lsum[kk] = s;
+      }
+#pragma unroll
+      for (int kk = 0; kk < NS; ++kk) lother[kk] = __shfl_xor_sync(0xffffffffu, lsum[kk], 1);
+      float* rec = v.partials + (size_t)(w + it.b * v.Hkv + it.h) * v.record_floats;
+      if (row == 0) {
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          float* oa = rec + g * D + DPC * j;
+          float* ob = rec + g * D + D / 2 + DPC * j;
+#pragma unroll
+          for (int e = 0; e < DPC; e += 4) {
+            *reinterpret_cast<float4*>(oa + e) = make_float4(o[g][e], o[g][e + 1], o[g][e + 2], o[g][e + 3]);
+            *reinterpret_cast<float4*>(ob + e) =
+                make_float4(o[g][DPC + e], o[g][DPC + e + 1], o[g][DPC + e + 2], o[g][DPC + e + 3]);
+          }
+        }
+      }
+      if (lane == 0) {
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          rec[G * D + g] = m_run[g];
+          rec[G * D + G + g] = ((g / NS) == b0) ? lsum[g % NS] : lother[g % NS];
+        }
+      }
+      fresh = true;
+    }
+    if (x + 1 < x_end) iter_advance(it, s_n, s_start, v.Hkv, v.max_beams);
+  }
+}
+
+// Merge the partial records of each (beam, kv head) into out[b][h*G+g][:].
+__global__ void k_combine(PoolView v, int mode, int W, float* __restrict__ out) {
+  const int bh = blockIdx.x;
+  const int b = bh / v.Hkv, h = bh % v.Hkv;
+  const int G = v.G, D = v.D;
+  float* ob = out + ((size_t)b * v.Hq + (size_t)h * G) * D;
+  const bool ok = v.ctl[kCtlStepOk] != 0 && v.active[b] != 0;
+  const int n = ok ? plan_n(v, mode)[b] : 0;
+  if (n == 0) {
+    for (int e = threadIdx.x; e < G * D; e += blockDim.x) ob[e] = 0.f;
+    return;
+  }
+  const int Tot = plan_off(v, mode)[v.max_beams];
+  const int c = (Tot + W - 1) / W;
+  const int off = plan_off(v, mode)[b] + h * n;
+  const int first = off / c, last = (off + n - 1) / c;
+  for (int e = threadIdx.x; e < G * D; e += blockDim.x) {
+    const int g = e / D;
+    float M = -INFINITY;
+    for (int w = first; w <= last; ++w) {
+      const float* rec = v.partials + (size_t)(w + bh) * v.record_floats;
+      M = fmaxf(M, rec[G * D + g]);
+    }
+    float l = 0.f, acc = 0.f;
+    for (int w = first; w <= last; ++w) {
+      const float* rec = v.partials + (size_t)(w + bh) * v.record_floats;
+      const float sc = exp2f(rec[G * D + g] - M);
+      l = fmaf(rec[G * D + G + g], sc, l);
+      acc = fmaf(rec[e], sc, acc);
+    }
+    ob[e] = acc / l;
+  }
+}
+
+template <int DT, int G>
+static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
+                                   cudaStream_t s) {
+  using S = DecodeSmem<DT, G>;
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(k_decode<DT, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, S::TOTAL);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  const int W = pool->decode_warps;
+  const float qscale = scale * 1.4426950408889634f;  // log2(e): softmax in base 2
+  k_decode<DT, G><<<W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s>>>(pool->view, layer, q, qscale, mode, W);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_combine<<<pool->view.max_beams * pool->view.Hkv, 128, 0, s>>>(pool->view, mode, W, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
+                          cudaStream_t s) {
+  const int G = pool->view.G;
+  if (pool->view.dtype == GB_BF16) {
+    switch (G) {
+      case 2: return launch_decode_t<GB_BF16, 2>(pool, layer, q, scale, out, mode, s);
+      case 4: return launch_decode_t<GB_BF16, 4>(pool, layer, q, scale, out, mode, s);
+      case 8: return launch_decode_t<GB_BF16, 8>(pool, layer, q, scale, out, mode, s);
+    }
+  } else {
+    switch (G) {
+      case 2: return launch_decode_t<GB_F32, 2>(pool, layer, q, scale, out, mode, s);
+      case 4: return launch_decode_t<GB_F32, 4>(pool, layer, q, scale, out, mode, s);
+      case 8: return launch_decode_t<GB_F32, 8>(pool, layer, q, scale, out, mode, s);
+    }
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace gb

@@ -1,0 +1,164 @@
+// Internal definitions shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <string>
+
+#include "gambit.h"
+
+namespace gb {
+
+constexpr int kMaxBeams = 1024;    // slots per pool (one thread per slot in the planners)
+constexpr int kChunk = 16;         // tokens per split-KV work unit (a page is 1..4 chunks)
+constexpr int kDecodeWarps = 8;    // warps per CTA of the split-KV decode kernel (one CTA per SM)
+constexpr int kDecodeStages = 3;   // TMA ring depth per warp
+constexpr int kDecodeCtasPerSm = 1;
+constexpr int kMaxDecodeWarps = 4096;
+constexpr int kMaxCowJobs = 1024;
+
+// Control words at the start of the metadata buffer.
+enum Ctl : int {
+  kCtlStatus = 0,      // first device-side error (GB_OK when none)
+  kCtlStepOk = 1,      // 1 while the current decode step has its pages
+  kCtlDone = 2,        // last-CTA-done ticket counter (reset by the last CTA)
+  kCtlCursor = 3,      // lowest free-bitmap word that may hold a free page
+  kCtlNextLineage = 4, // next lineage id to hand out
+  kCtlFree = 5,        // number of free pages
+  kCtlWords = 32
+};
+
+// Byte offsets of the metadata regions.
+struct MetaLayout {
+  size_t ctl, tables, seq_len, active, gen, nsteps, mean, lineage, refcnt, free_bits;
+  size_t plan, partials, total;
+  int words;            // free-bitmap words
+  int partial_records;  // split-KV partial records
+  int record_floats;    // floats per partial record: G*(D+2)
+};
+
+MetaLayout meta_layout(const gb_pool_config& c);
+
+// Plain-old-data view of a pool passed by value to kernels.
+struct PoolView {
+  int layers, Hq, Hkv, D, P, G, dtype, esize, max_beams, max_pages, words;
+  long long num_pages;
+  char* kv;             // KV pool base
+  long long page_elems; // elements of one (layer, page): 2*Hkv*P*D
+  int* ctl;
+  int* tables;          // [max_beams][max_pages]
+  int* seq_len;
+  int* active;
+  int* gen;
+  int* nsteps;
+  float* mean;
+  unsigned* lineage;
+  int* refcnt;
+  unsigned* free_bits;
+  int* plan;            // [2 modes][3][max_beams + 1]: offsets, chunk counts, start tokens
+  float* partials;
+  int record_floats;
+};
+
+// Plan arrays: mode 0 = per-beam only, mode 1 = with grouped coverage.
+__host__ __device__ inline int* plan_off(const PoolView& v, int mode) {
+  return v.plan + (size_t)mode * 3 * (v.max_beams + 1);
+}
+__host__ __device__ inline int* plan_n(const PoolView& v, int mode) {
+  return plan_off(v, mode) + (v.max_beams + 1);
+}
+__host__ __device__ inline int* plan_start(const PoolView& v, int mode) {
+  return plan_off(v, mode) + 2 * (v.max_beams + 1);
+}
+
+// Element offset of row `row` of the K (kv=0) or V (kv=1) slab of (layer, page, head).
+__device__ __forceinline__ long long kv_elem_offset(const PoolView& v, int layer, long long page,
+                                                    int kv, int head, int row) {
+  return ((((long long)layer * v.num_pages + page) * 2 + kv) * v.Hkv + head) * (long long)v.P * v.D +
+         (long long)row * v.D;
+}
+
+__device__ __forceinline__ void set_status(int* ctl, int code) {
+  atomicCAS(&ctl[kCtlStatus], GB_OK, code);
+}
+
+// Mark page p free (bitmap, allocation cursor, free count).
+__device__ __forceinline__ void mark_free(const PoolView& v, int p) {
+  atomicOr(&v.free_bits[p >> 5], 1u << (p & 31));
+  atomicMin(&v.ctl[kCtlCursor], p >> 5);
+  atomicAdd(&v.ctl[kCtlFree], 1);
+}
+
+// Drop one reference to page p; frees it when the count reaches zero.
+__device__ __forceinline__ void unref_page(const PoolView& v, int p) {
+  if (atomicSub(&v.refcnt[p], 1) == 1) mark_free(v, p);
+}
+
+// Block-wide exclusive scan of one int per thread (blockDim.x <= 1024, multiple of 32).
+// `tmp` must hold 33 ints of shared memory.  Returns the exclusive prefix; *total gets the sum.
+__device__ __forceinline__ int block_exclusive_scan(int x, int* tmp, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  int inc = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    int y = __shfl_up_sync(0xffffffffu, inc, o);
+    if (lane >= o) inc += y;
+  }
+  if (lane == 31) tmp[warp] = inc;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < nwarps ? tmp[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < nwarps) tmp[lane] = w;  // inclusive warp totals
+    if (lane == nwarps - 1) tmp[32] = w;
+  }
+  __syncthreads();
+  int r = inc - x + (warp > 0 ? tmp[warp - 1] : 0);
+  *total = tmp[32];
+  __syncthreads();
+  return r;
+}
+
+// Host side --------------------------------------------------------------------
+
+struct DecodeShape {
+  int dtype, D, G;
+};
+bool decode_supported(int dtype, int D, int G);
+
+}  // namespace gb
+
+// The opaque host handle.
+struct gb_pool {
+  gb_pool_config cfg;
+  gb::MetaLayout layout;
+  gb::PoolView view;
+  int device;
+  int num_sms;
+  int decode_warps;   // warps launched by the split-KV decode kernel
+  int next_layer;     // layer expected by the next decode/append call (0 opens a step)
+  int step_tokens;    // tokens reserved by the open step
+  bool seeded;
+  int group_min;
+  std::string last_error;
+};
+
+namespace gb {
+gb_status fail(gb_pool* pool, gb_status code, const char* what);
+gb_status check_launch(gb_pool* pool, const char* what);
+
+// Kernel launchers implemented in the other translation units.
+cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
+                          cudaStream_t s);
+cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
+                         float bias, const uint8_t* mask, float* score_out, const float* scores_in,
+                         cudaStream_t s);
+cudaError_t launch_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const uint8_t* elig,
+                                int32_t* parent_out, uint8_t* pruned_out, uint32_t* lineage_out,
+                                cudaStream_t s);
+}  // namespace gb
