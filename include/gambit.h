@@ -225,6 +225,25 @@ gb_status gb_pool_clear_status(gb_pool* pool, gb_stream_t stream);
 /* Synchronise `stream` and copy the pool state into host arrays (see gb_pool_state). */
 gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_stream_t stream);
 
+/*
+ * Instrumentation (not part of the method).  Record caller-created CUDA
+ * events (cudaEvent_t) immediately before and after one kernel of the
+ * following calls on this pool, so a caller can time that kernel alone on its
+ * own stream: `which` is GB_PROF_DECODE (the split-KV decode kernel of
+ * gb_decode_attention), GB_PROF_PROBE (gb_score_probe) or GB_PROF_PRUNE
+ * (gb_prune_branch).  Passing NULL events stops recording.  The events stay
+ * owned by the caller.
+ */
+#define GB_PROF_DECODE 0
+#define GB_PROF_PROBE 1
+#define GB_PROF_PRUNE 2
+#define GB_PROF_GROUPED 3
+#define GB_PROF_SLOTS 4
+gb_status gb_pool_set_profile_events(gb_pool* pool, int which, void* start_event, void* stop_event);
+
+/* Number of kernels this pool has launched since gb_pool_init (host-side count). */
+gb_status gb_pool_launch_count(gb_pool* pool, uint64_t* count);
+
 /* Short description of the pool's last host-side failure ("" if none); static storage. */
 const char* gb_last_error(gb_pool* pool);
 

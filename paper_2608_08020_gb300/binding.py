@@ -25,7 +25,9 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 # Every symbol the header declares, in header order.
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
-           "gb_pool_clear_status", "gb_pool_read_state", "gb_last_error"]
+           "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
+           "gb_last_error"]
+GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
 
 
 class GbPoolConfig(ctypes.Structure):
@@ -74,6 +76,8 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_pool_status": [V, P, V],
         "gb_pool_clear_status": [V, V],
         "gb_pool_read_state": [V, P, V],
+        "gb_pool_set_profile_events": [V, I, V, V],
+        "gb_pool_launch_count": [V, P],
         "gb_last_error": [V],
     }
     for name, args in sig.items():
@@ -183,6 +187,22 @@ def gb_pool_clear_status(pool: int, stream=None) -> None:
 
 def gb_pool_read_state(pool: int, state: GbPoolState, stream=None) -> None:
     _check(pool, load().gb_pool_read_state(pool, ctypes.byref(state), stream_handle(stream)), "gb_pool_read_state")
+
+
+def gb_pool_set_profile_events(pool: int, which: int, start_event=None, stop_event=None) -> None:
+    """Events may be torch.cuda.Event objects (already recorded once) or raw cudaEvent_t ints."""
+    def ev(e):
+        if e is None or isinstance(e, int):
+            return e
+        return e.cuda_event
+    _check(pool, load().gb_pool_set_profile_events(pool, which, ev(start_event), ev(stop_event)),
+           "gb_pool_set_profile_events")
+
+
+def gb_pool_launch_count(pool: int) -> int:
+    n = ctypes.c_uint64()
+    _check(pool, load().gb_pool_launch_count(pool, ctypes.byref(n)), "gb_pool_launch_count")
+    return n.value
 
 
 def gb_last_error(pool: int) -> str:

@@ -442,10 +442,13 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
   }
   const int W = pool->decode_warps;
   const float qscale = scale * 1.4426950408889634f;  // log2(e): softmax in base 2
+  prof_begin(pool, GB_PROF_DECODE, s);
   k_decode<DT, G><<<W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s>>>(pool->view, layer, q, qscale, mode, W);
+  prof_end(pool, GB_PROF_DECODE, s);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   k_combine<<<pool->view.max_beams * pool->view.Hkv, 128, 0, s>>>(pool->view, mode, W, out);
+  pool->launches += 2;
   return cudaGetLastError();
 }
 

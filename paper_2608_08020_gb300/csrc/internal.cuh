@@ -146,10 +146,21 @@ struct gb_pool {
   bool seeded;
   int group_min;
   std::string last_error;
+  unsigned long long launches = 0;          // kernels launched by this pool
+  cudaEvent_t prof_start[GB_PROF_SLOTS] = {};  // caller-owned instrumentation events
+  cudaEvent_t prof_stop[GB_PROF_SLOTS] = {};
 };
 
 namespace gb {
 gb_status fail(gb_pool* pool, gb_status code, const char* what);
+
+// Instrumentation: record the caller's event pair around one kernel, if set.
+inline void prof_begin(gb_pool* p, int which, cudaStream_t s) {
+  if (p->prof_start[which]) cudaEventRecord(p->prof_start[which], s);
+}
+inline void prof_end(gb_pool* p, int which, cudaStream_t s) {
+  if (p->prof_stop[which]) cudaEventRecord(p->prof_stop[which], s);
+}
 gb_status check_launch(gb_pool* pool, const char* what);
 
 // Kernel launchers implemented in the other translation units.

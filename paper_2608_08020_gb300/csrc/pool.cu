@@ -450,6 +450,7 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
     delete p;
     return GB_ERR_CUDA;
   }
+  p->launches += 1;
   k_init<<<std::max(1, std::min(p->num_sms * 4, (int)((v.max_beams * (long long)v.max_pages + 255) / 256))), 256, 0, s>>>(v);
   st = check_launch(p, "init");
   if (st != GB_OK) {
@@ -479,6 +480,7 @@ extern "C" gb_status gb_pool_seed(gb_pool* pool, int n_beams, int prompt_len, co
     return fail(pool, GB_ERR_UNSUPPORTED, "seed: prompt longer than 2048 pages");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   k_seed_alloc<<<1, 1024, 0, s>>>(pool->view, n_beams, prompt_len);
+  pool->launches += 2;
   gb_status st = check_launch(pool, "seed_alloc");
   if (st != GB_OK) return st;
   const long long vecs = 2LL * pool->cfg.num_layers * prompt_len * pool->cfg.num_kv_heads *
@@ -503,6 +505,7 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
   if (layer != pool->next_layer) return fail(pool, GB_ERR_STATE, "layers of a step must be called in order");
   if (layer == 0) {
     k_step_begin<<<1, 1024, 0, s>>>(pool->view, n_tokens, nullptr);
+    pool->launches += 1;
     gb_status st = check_launch(pool, "step_begin");
     if (st != GB_OK) return st;
     pool->step_tokens = n_tokens;
@@ -514,6 +517,7 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
   const int grid = (int)std::min<long long>((vecs + 255) / 256, pool->num_sms * 8LL);
   k_append<<<std::max(grid, 1), 256, 0, s>>>(pool->view, layer, n_tokens, static_cast<const char*>(k),
                                              static_cast<const char*>(v));
+  pool->launches += 1;
   gb_status st = check_launch(pool, "append");
   if (st != GB_OK) return st;
   pool->next_layer = (layer + 1) % pool->cfg.num_layers;
@@ -547,6 +551,7 @@ extern "C" gb_status gb_release(gb_pool* pool, const int32_t* slots_dev, int n, 
   if (pool->next_layer != 0) return fail(pool, GB_ERR_STATE, "release inside an open step");
   if (n == 0) return GB_OK;
   k_release<<<1, 1024, 0, reinterpret_cast<cudaStream_t>(stream)>>>(pool->view, slots_dev, n);
+  pool->launches += 1;
   return check_launch(pool, "release");
 }
 
@@ -561,9 +566,23 @@ extern "C" gb_status gb_pool_status(gb_pool* pool, int* device_status, gb_stream
   return GB_OK;
 }
 
+extern "C" gb_status gb_pool_set_profile_events(gb_pool* pool, int which, void* start_event, void* stop_event) {
+  if (!pool || which < 0 || which >= GB_PROF_SLOTS) return GB_ERR_INVALID;
+  pool->prof_start[which] = static_cast<cudaEvent_t>(start_event);
+  pool->prof_stop[which] = static_cast<cudaEvent_t>(stop_event);
+  return GB_OK;
+}
+
+extern "C" gb_status gb_pool_launch_count(gb_pool* pool, uint64_t* count) {
+  if (!pool || !count) return GB_ERR_INVALID;
+  *count = pool->launches;
+  return GB_OK;
+}
+
 extern "C" gb_status gb_pool_clear_status(gb_pool* pool, gb_stream_t stream) {
   if (!pool) return GB_ERR_INVALID;
   k_clear_status<<<1, 1, 0, reinterpret_cast<cudaStream_t>(stream)>>>(pool->view);
+  pool->launches += 1;
   return check_launch(pool, "clear_status");
 }
 

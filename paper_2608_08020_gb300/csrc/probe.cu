@@ -75,10 +75,13 @@ cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, in
                          const uint8_t* mask, float* score_out, const float* scores_in, cudaStream_t s) {
   const int warps_per_block = 8;
   const int grid = (pool->view.max_beams + warps_per_block - 1) / warps_per_block;
+  pool->launches += 1;
+  if (scores_in == nullptr) prof_begin(pool, GB_PROF_PROBE, s);
   if (hidden_dtype == GB_BF16)
     k_probe<GB_BF16><<<grid, warps_per_block * 32, 0, s>>>(pool->view, hidden, H, w, bias, mask, score_out, scores_in);
   else
     k_probe<GB_F32><<<grid, warps_per_block * 32, 0, s>>>(pool->view, hidden, H, w, bias, mask, score_out, scores_in);
+  if (scores_in == nullptr) prof_end(pool, GB_PROF_PROBE, s);
   return cudaGetLastError();
 }
 

@@ -164,8 +164,11 @@ __global__ void __launch_bounds__(1024) k_prune_branch(PoolView v, int K, int fa
 cudaError_t launch_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const uint8_t* elig,
                                 int32_t* parent_out, uint8_t* pruned_out, uint32_t* lineage_out, cudaStream_t s) {
   const int grid = pool->view.max_beams < pool->num_sms ? pool->view.max_beams : pool->num_sms;
+  prof_begin(pool, GB_PROF_PRUNE, s);
   k_prune_branch<<<grid, 1024, 0, s>>>(pool->view, K, fanout, warmup, elig, parent_out, pruned_out,
                                        reinterpret_cast<unsigned*>(lineage_out));
+  prof_end(pool, GB_PROF_PRUNE, s);
+  pool->launches += 1;
   return cudaGetLastError();
 }
 
