@@ -220,7 +220,7 @@ def run_ours(args) -> None:
     W, K = args.warmup, args.steps
     S = W + 2 * K
 
-    g = GpuRun(wl, device_gen=True, device=str(dev))
+    g = GpuRun(wl, device_gen=True, device=str(dev), max_context=wl.context + S + 1)
     t_build = time.perf_counter()
     g.build(upto=wl.context)
     torch.cuda.synchronize()
@@ -299,6 +299,8 @@ def run_ours(args) -> None:
     prune_us = statistics.mean(a.elapsed_time(b) for a, b in zip(pr_a, pr_b)) * 1e3
     probe_us = statistics.mean(a.elapsed_time(b) for a, b in zip(pb_a, pb_b)) * 1e3
     status = pool.status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after the timed steps: the measurement is invalid")
 
     # Algorithmic bytes of one decode-kernel launch: every beam's K and V once, plus its queries.
     kv_tok = 2 * Hkv * D * (2 if wl.kv_dtype == "bf16" else 4)

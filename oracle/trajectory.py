@@ -23,10 +23,11 @@ from workload.configs import Workload
 
 
 class OracleRun:
-    def __init__(self, wl: Workload, literal_kv: bool = True, num_pages: int | None = None):
+    def __init__(self, wl: Workload, literal_kv: bool = True, num_pages: int | None = None,
+                 max_context: int | None = None):
         self.wl = wl
-        self.pool = PoolOracle(num_pages if num_pages is not None else wl.pool_pages(), wl.beams,
-                               wl.pages_per_beam + 1, wl.page_size)
+        self.pool = PoolOracle(num_pages if num_pages is not None else wl.pool_pages(max_context), wl.beams,
+                               wl.table_width(max_context), wl.page_size)
         self.kv = BeamKV(wl.num_layers, wl.beams, wl.num_kv_heads, wl.head_dim) if literal_kv else None
         self.hscale = None
         if wl.head_scale is not None:

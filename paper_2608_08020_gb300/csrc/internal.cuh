@@ -26,13 +26,14 @@ enum Ctl : int {
   kCtlCursor = 3,      // lowest free-bitmap word that may hold a free page
   kCtlNextLineage = 4, // next lineage id to hand out
   kCtlFree = 5,        // number of free pages
+  kCtlCowJobs = 6,     // copy-on-write jobs of the open step (rows copied by each layer's append)
   kCtlWords = 32
 };
 
 // Byte offsets of the metadata regions.
 struct MetaLayout {
   size_t ctl, tables, seq_len, active, gen, nsteps, mean, lineage, refcnt, free_bits;
-  size_t plan, partials, total;
+  size_t plan, cow, partials, total;
   int words;            // free-bitmap words
   int partial_records;  // split-KV partial records
   int record_floats;    // floats per partial record: G*(D+2)
@@ -57,6 +58,7 @@ struct PoolView {
   int* refcnt;
   unsigned* free_bits;
   int* plan;            // [2 modes][3][max_beams + 1]: offsets, chunk counts, start tokens
+  int* cow;             // [kMaxCowJobs][3] (old page, new page, rows) of the open step's copy-on-writes
   float* partials;
   int record_floats;
 };

@@ -33,6 +33,7 @@ MetaLayout meta_layout(const gb_pool_config& c) {
   m.words = (int)((c.num_pages + 31) / 32);
   m.free_bits = take((size_t)m.words * sizeof(unsigned));
   m.plan = take(2 * 3 * (B + 1) * sizeof(int));
+  m.cow = take(kMaxCowJobs * 3 * sizeof(int));
   m.record_floats = G * (c.head_dim + 2);
   m.partial_records = kMaxDecodeWarps + (int)B * c.num_kv_heads;
   m.partials = take((size_t)m.partial_records * m.record_floats * sizeof(float));
@@ -185,7 +186,6 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
   __shared__ int tmp[33];
   __shared__ int s_alloc[kMaxBeams];
   __shared__ int s_tail[kMaxBeams];
-  __shared__ int s_cow_old[kMaxCowJobs], s_cow_new[kMaxCowJobs], s_cow_rows[kMaxCowJobs];
   __shared__ int s_ncow;
   const int b = threadIdx.x;
   const bool act = b < v.max_beams && v.active[b] != 0;
@@ -221,6 +221,7 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
   block_exclusive_scan(need_total, tmp, &total_need);
   const bool any_too_long = __syncthreads_or(too_long);
   if (any_too_long || total_need > v.ctl[kCtlFree]) {
+    if (b == 0) v.ctl[kCtlCowJobs] = 0;
     if (b == 0) { set_status(v.ctl, GB_ERR_OOM); v.ctl[kCtlStepOk] = 0; }
     return;
   }
@@ -246,33 +247,16 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
         atomicSub(&v.refcnt[tail], 1);
         const int j = atomicAdd(&s_ncow, 1);
         if (j < kMaxCowJobs) {
-          s_cow_old[j] = tail; s_cow_new[j] = page; s_cow_rows[j] = L % v.P;
+          v.cow[3 * j] = tail;
+          v.cow[3 * j + 1] = page;
+          v.cow[3 * j + 2] = L % v.P;
         }
       }
     }
     __syncthreads();
-    if (k == 0 && s_ncow > 0) {
-      // Copy rows [0, rows) of every layer, K and V, every head, old page -> new page.
-      const int ncow = min(s_ncow, kMaxCowJobs);
-      const int vec_per_row = v.D * v.esize / 16;
-      const long long per_job = (long long)v.layers * 2 * v.Hkv * v.P * vec_per_row;
-      for (long long i = threadIdx.x; i < per_job * ncow; i += blockDim.x) {
-        const int j = (int)(i / per_job);
-        long long r = i % per_job;
-        const int vec = (int)(r % vec_per_row); r /= vec_per_row;
-        const int row = (int)(r % v.P); r /= v.P;
-        if (row >= s_cow_rows[j]) continue;
-        const int head = (int)(r % v.Hkv); r /= v.Hkv;
-        const int kv = (int)(r % 2);
-        const int layer = (int)(r / 2);
-        const uint4* src = reinterpret_cast<const uint4*>(
-            v.kv + kv_elem_offset(v, layer, s_cow_old[j], kv, head, row) * v.esize);
-        uint4* dst = reinterpret_cast<uint4*>(v.kv + kv_elem_offset(v, layer, s_cow_new[j], kv, head, row) * v.esize);
-        dst[vec] = src[vec];
-      }
-      __syncthreads();
-    }
   }
+  // The rows [0, L % P) of each copied page are copied layer by layer by the append kernel.
+  if (b == 0) v.ctl[kCtlCowJobs] = min(s_ncow, kMaxCowJobs);
 
   const int Lnew = act ? L + n_tokens : 0;
   if (act) {
@@ -303,6 +287,23 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
 __global__ void k_append(PoolView v, int layer, int n_tokens, const char* kin, const char* vin) {
   if (v.ctl[kCtlStepOk] == 0) return;
   const int vec_per_row = v.D * v.esize / 16;
+  // Copy-on-write of still-shared partial tail pages, this layer's rows [0, rows).
+  // Rows differ from every row written below, so both loops run concurrently.
+  const int ncow = v.ctl[kCtlCowJobs];
+  const long long per_job = 2LL * v.Hkv * v.P * vec_per_row;
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_job * ncow;
+       i += (long long)gridDim.x * blockDim.x) {
+    const int j = (int)(i / per_job);
+    long long r = i % per_job;
+    const int vec = (int)(r % vec_per_row); r /= vec_per_row;
+    const int row = (int)(r % v.P); r /= v.P;
+    if (row >= v.cow[3 * j + 2]) continue;
+    const int head = (int)(r % v.Hkv);
+    const int kv = (int)(r / v.Hkv);
+    const uint4* src = reinterpret_cast<const uint4*>(v.kv + kv_elem_offset(v, layer, v.cow[3 * j], kv, head, row) * v.esize);
+    uint4* dst = reinterpret_cast<uint4*>(v.kv + kv_elem_offset(v, layer, v.cow[3 * j + 1], kv, head, row) * v.esize);
+    dst[vec] = src[vec];
+  }
   const long long per_tok = (long long)v.max_beams * v.Hkv * vec_per_row;
   const long long total = per_tok * n_tokens * 2;
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
@@ -443,6 +444,7 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   v.refcnt = reinterpret_cast<int*>(m + L.refcnt);
   v.free_bits = reinterpret_cast<unsigned*>(m + L.free_bits);
   v.plan = reinterpret_cast<int*>(m + L.plan);
+  v.cow = reinterpret_cast<int*>(m + L.cow);
   v.partials = reinterpret_cast<float*>(m + L.partials);
   v.record_floats = L.record_floats;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

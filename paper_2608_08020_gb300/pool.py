@@ -31,12 +31,13 @@ class BeamPool:
         self.handle = B.gb_pool_init(self.cfg, self.kv, self.meta, stream)
 
     @classmethod
-    def for_workload(cls, wl, device="cuda", num_pages: int | None = None, group_min_beams: int = 0, max_beams=None):
+    def for_workload(cls, wl, device="cuda", num_pages: int | None = None, group_min_beams: int = 0, max_beams=None,
+                     max_context: int | None = None):
         return cls(num_layers=wl.num_layers, num_q_heads=wl.num_q_heads, num_kv_heads=wl.num_kv_heads,
                    head_dim=wl.head_dim, page_size=wl.page_size, kv_dtype=wl.kv_dtype,
-                   num_pages=num_pages if num_pages is not None else wl.pool_pages(),
+                   num_pages=num_pages if num_pages is not None else wl.pool_pages(max_context),
                    max_beams=max_beams if max_beams is not None else wl.beams,
-                   max_pages_per_beam=wl.pages_per_beam + 1, group_min_beams=group_min_beams, device=device)
+                   max_pages_per_beam=wl.table_width(max_context), group_min_beams=group_min_beams, device=device)
 
     def close(self) -> None:
         if self.handle:

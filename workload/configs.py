@@ -59,19 +59,23 @@ class Workload:
     def pages_per_beam(self) -> int:
         return -(-self.context // self.page_size)
 
+    def table_width(self, max_context: int | None = None) -> int:
+        """Block-table entries per slot for contexts up to max_context (default: the workload's)."""
+        return -(-(max_context or self.context) // self.page_size) + 1
+
     def kv_bytes_per_token_layer(self) -> int:
         return 2 * self.num_kv_heads * self.head_dim * self.esize
 
     def page_bytes_all_layers(self) -> int:
         return self.num_layers * self.page_size * self.kv_bytes_per_token_layer()
 
-    def pool_pages(self) -> int:
+    def pool_pages(self, max_context: int | None = None) -> int:
         if self.num_pages is not None:
             return self.num_pages
         if self.pool_bytes is not None:
             return self.pool_bytes // self.page_bytes_all_layers()
         # Enough for every beam to hold its whole context unshared, plus slack.
-        return self.beams * (self.pages_per_beam + 1) + 64
+        return self.beams * (self.table_width(max_context) + 1) + 64
 
     def rounds(self, include_final: bool = False) -> list[int]:
         """Context lengths at which probe + tournament run during the build."""

@@ -22,11 +22,12 @@ from workload.configs import Workload
 
 class GpuRun:
     def __init__(self, wl: Workload, device_gen: bool = False, device: str = "cuda", num_pages: int | None = None,
-                 group_min_beams: int = 0, max_chunk: int = 256):
+                 group_min_beams: int = 0, max_chunk: int = 256, max_context: int | None = None):
         self.wl = wl
         self.device_gen = device_gen
         self.dev = torch.device(device)
-        self.pool = BeamPool.for_workload(wl, device=device, num_pages=num_pages, group_min_beams=group_min_beams)
+        self.pool = BeamPool.for_workload(wl, device=device, num_pages=num_pages, group_min_beams=group_min_beams,
+                                          max_context=max_context)
         C, Hq, Hkv, D = wl.beams, wl.num_q_heads, wl.num_kv_heads, wl.head_dim
         self.C = C
         self.tdt = TORCH_DT[wl.kv_dtype]
