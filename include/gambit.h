@@ -244,6 +244,64 @@ gb_status gb_pool_set_profile_events(gb_pool* pool, int which, void* start_event
 /* Number of kernels this pool has launched since gb_pool_init (host-side count). */
 gb_status gb_pool_launch_count(gb_pool* pool, uint64_t* count);
 
+/*
+ * Decode attention over caller-managed pages that allocates nothing.
+ *
+ * The paper has no counterpart; this entry point exists for callers that cannot
+ * allocate device memory where they decode - for example a serving process whose
+ * allocator takes the GPU's memory when it starts and allows no allocation on the
+ * token path, or code running inside a framework whose device memory it does not
+ * own.  The caller passes only inputs and outputs; the call's working memory (work
+ * plan and split-KV partial results) is a fixed 32 MiB array in the library's own
+ * device memory, which every GPU that loads the library holds until the process
+ * exits.  No cudaMalloc, cudaFree or allocating library routine is called.
+ *
+ * Computes, for every row b with seq_len[b] > 0 and query head h,
+ *   out[b][h] = sum_t softmax_t(scale * q[b][h] . K_b[t]) V_b[t],  t in [0, seq_len[b])
+ * where token t of row b is row t % page_size of page tables[b][t / page_size] and
+ * query head h reads KV head h / (num_q_heads / num_kv_heads).  Rows with
+ * seq_len[b] == 0 give zeros.  Arguments (device pointers):
+ *   kv:      one layer's pages, [num_pages][K|V][num_kv_heads][page_size][head_dim] in
+ *            kv_dtype (the layout of a gb_pool layer), 16-byte aligned
+ *   tables:  int32 [num_beams][max_pages_per_beam];  seq_len: int32 [num_beams]
+ *   q:       [num_beams][num_q_heads][head_dim] in kv_dtype, 16-byte aligned
+ *   out:     fp32 [num_beams][num_q_heads][head_dim]
+ * Page ids are trusted: an id outside [0, num_pages) is not dereferenced (page 0 is
+ * read in its place) and that row's output is unspecified.
+ *
+ * The scratch array is shared by every call on a device and keeps the last call's
+ * contents; each call rewrites all of it that it reads, and clears its own status
+ * word.  Calls whose GPU work overlaps (different streams, or host threads issuing
+ * concurrently) race on it: keep them ordered, e.g. on one stream.
+ * The first call on a device looks up the array's device address with
+ * cudaGetSymbolAddress (with that device current); that first call should come
+ * before any stream capture.
+ * Errors: GB_ERR_INVALID for bad shapes or null/misaligned pointers,
+ * GB_ERR_UNSUPPORTED for a (kv_dtype, head_dim, Hq/Hkv) without a kernel, and
+ * GB_ERR_TOO_LARGE when the scratch needed, 256-byte rounded
+ *   128 + 4*num_beams + 12*(num_beams+1) + 4*(W + num_beams*num_kv_heads)*G*(head_dim+2)
+ * bytes with W = 8 x (multiprocessor count) and G = num_q_heads/num_kv_heads, exceeds 32 MiB
+ * (for G = 4, head_dim 128 and 8 KV heads: up to 1024 rows on a 152-SM GB300).
+ */
+#define GB_ERR_TOO_LARGE 7  /* the call needs more fixed scratch than the library holds */
+typedef struct {
+  const void* kv;
+  const int32_t* tables;
+  const int32_t* seq_len;
+  const void* q;
+  float* out;
+  int num_beams;
+  int num_q_heads;
+  int num_kv_heads;
+  int head_dim;
+  int page_size;
+  int kv_dtype;
+  int max_pages_per_beam;
+  int64_t num_pages;
+  float scale;
+} gb_paged_decode_args;
+gb_status gb_paged_decode_noalloc(const gb_paged_decode_args* args, gb_stream_t stream);
+
 /* Short description of the pool's last host-side failure ("" if none); static storage. */
 const char* gb_last_error(gb_pool* pool);
 

@@ -17,8 +17,9 @@ from pathlib import Path
 LIB_PATH = Path(__file__).resolve().with_name("libgambit.so")
 
 GB_OK, GB_ERR_INVALID, GB_ERR_OOM, GB_ERR_CUDA, GB_ERR_STATE, GB_ERR_TIMEOUT, GB_ERR_UNSUPPORTED = range(7)
+GB_ERR_TOO_LARGE = 7
 STATUS_NAMES = {0: "GB_OK", 1: "GB_ERR_INVALID", 2: "GB_ERR_OOM", 3: "GB_ERR_CUDA", 4: "GB_ERR_STATE",
-                5: "GB_ERR_TIMEOUT", 6: "GB_ERR_UNSUPPORTED"}
+                5: "GB_ERR_TIMEOUT", 6: "GB_ERR_UNSUPPORTED", 7: "GB_ERR_TOO_LARGE"}
 GB_F32, GB_BF16 = 0, 1
 GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 
@@ -26,7 +27,7 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
            "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
-           "gb_last_error"]
+           "gb_paged_decode_noalloc", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
 
 
@@ -41,6 +42,14 @@ class GbPoolState(ctypes.Structure):
     _fields_ = [("tables", ctypes.c_void_p), ("seq_len", ctypes.c_void_p), ("active", ctypes.c_void_p),
                 ("gen", ctypes.c_void_p), ("nsteps", ctypes.c_void_p), ("mean", ctypes.c_void_p),
                 ("lineage", ctypes.c_void_p), ("refcnt", ctypes.c_void_p), ("free_bits", ctypes.c_void_p)]
+
+
+class GbPagedDecodeArgs(ctypes.Structure):
+    _fields_ = [("kv", ctypes.c_void_p), ("tables", ctypes.c_void_p), ("seq_len", ctypes.c_void_p),
+                ("q", ctypes.c_void_p), ("out", ctypes.c_void_p), ("num_beams", ctypes.c_int),
+                ("num_q_heads", ctypes.c_int), ("num_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int),
+                ("page_size", ctypes.c_int), ("kv_dtype", ctypes.c_int), ("max_pages_per_beam", ctypes.c_int),
+                ("num_pages", ctypes.c_int64), ("scale", ctypes.c_float)]
 
 
 class GambitError(RuntimeError):
@@ -78,6 +87,7 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_pool_read_state": [V, P, V],
         "gb_pool_set_profile_events": [V, I, V, V],
         "gb_pool_launch_count": [V, P],
+        "gb_paged_decode_noalloc": [P, V],
         "gb_last_error": [V],
     }
     for name, args in sig.items():
@@ -203,6 +213,12 @@ def gb_pool_launch_count(pool: int) -> int:
     n = ctypes.c_uint64()
     _check(pool, load().gb_pool_launch_count(pool, ctypes.byref(n)), "gb_pool_launch_count")
     return n.value
+
+
+def gb_paged_decode_noalloc(args: GbPagedDecodeArgs, stream=None) -> None:
+    """Paged decode attention with the library's fixed scratch (no allocation, no workspace)."""
+    _check(None, load().gb_paged_decode_noalloc(ctypes.byref(args), stream_handle(stream)),
+           "gb_paged_decode_noalloc")
 
 
 def gb_last_error(pool: int) -> str:

@@ -452,6 +452,44 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
   return cudaGetLastError();
 }
 
+// Split-KV decode + combine on an explicit view (plan mode 0, W warps), for callers
+// that supply their own tables and scratch instead of a pool.
+template <int DT, int G>
+static cudaError_t launch_view_t(const PoolView& v, int W, int layer, const void* q, float scale, float* out,
+                                 cudaStream_t s) {
+  using S = DecodeSmem<DT, G>;
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(k_decode<DT, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, S::TOTAL);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  const float qscale = scale * 1.4426950408889634f;
+  k_decode<DT, G><<<W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s>>>(v, layer, q, qscale, 0, W);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_combine<<<v.max_beams * v.Hkv, 128, 0, s>>>(v, 0, W, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* q, float scale, float* out,
+                               cudaStream_t s) {
+  if (v.dtype == GB_BF16) {
+    switch (v.G) {
+      case 2: return launch_view_t<GB_BF16, 2>(v, W, layer, q, scale, out, s);
+      case 4: return launch_view_t<GB_BF16, 4>(v, W, layer, q, scale, out, s);
+      case 8: return launch_view_t<GB_BF16, 8>(v, W, layer, q, scale, out, s);
+    }
+  } else {
+    switch (v.G) {
+      case 2: return launch_view_t<GB_F32, 2>(v, W, layer, q, scale, out, s);
+      case 4: return launch_view_t<GB_F32, 4>(v, W, layer, q, scale, out, s);
+      case 8: return launch_view_t<GB_F32, 8>(v, W, layer, q, scale, out, s);
+    }
+  }
+  return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
                           cudaStream_t s) {
   const int G = pool->view.G;

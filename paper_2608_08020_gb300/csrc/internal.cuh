@@ -168,6 +168,8 @@ gb_status check_launch(gb_pool* pool, const char* what);
 // Kernel launchers implemented in the other translation units.
 cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
                           cudaStream_t s);
+cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* q, float scale, float* out,
+                               cudaStream_t s);
 cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
                          float bias, const uint8_t* mask, float* score_out, const float* scores_in,
                          cudaStream_t s);
