@@ -396,7 +396,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
   }
 }
 
-// Merge the partial records of each (beam, kv head) into out[b][h*G+g][:].
+// Merge the partial records of each (beam, kv head) into out[b][h*G+g][:]: the split-KV
+// records of the warps that covered the beam's per-beam range and, in mode 1, the grouped
+// records of the beam's shared-prefix segments.
 __global__ void k_combine(PoolView v, int mode, int W, float* __restrict__ out) {
   const int bh = blockIdx.x;
   const int b = bh / v.Hkv, h = bh % v.Hkv;
@@ -404,24 +406,31 @@ __global__ void k_combine(PoolView v, int mode, int W, float* __restrict__ out) 
   float* ob = out + ((size_t)b * v.Hq + (size_t)h * G) * D;
   const bool ok = v.ctl[kCtlStepOk] != 0 && v.active[b] != 0;
   const int n = ok ? plan_n(v, mode)[b] : 0;
-  if (n == 0) {
+  const int nseg = (ok && mode == 1 && v.grouped) ? v.seg_nseg[b] : 0;
+  if (n == 0 && nseg == 0) {
     for (int e = threadIdx.x; e < G * D; e += blockDim.x) ob[e] = 0.f;
     return;
   }
   const int Tot = plan_off(v, mode)[v.max_beams];
-  const int c = (Tot + W - 1) / W;
+  const int c = Tot > 0 ? (Tot + W - 1) / W : 1;
   const int off = plan_off(v, mode)[b] + h * n;
-  const int first = off / c, last = (off + n - 1) / c;
+  const int first = off / c, last = n > 0 ? (off + n - 1) / c : first - 1;
+  const float* grec = v.grec + ((size_t)b * kMaxSegDepth * v.Hkv + h) * v.record_floats;
+  const size_t gstride = (size_t)v.Hkv * v.record_floats;
   for (int e = threadIdx.x; e < G * D; e += blockDim.x) {
     const int g = e / D;
     float M = -INFINITY;
-    for (int w = first; w <= last; ++w) {
-      const float* rec = v.partials + (size_t)(w + bh) * v.record_floats;
-      M = fmaxf(M, rec[G * D + g]);
-    }
+    for (int w = first; w <= last; ++w) M = fmaxf(M, v.partials[(size_t)(w + bh) * v.record_floats + G * D + g]);
+    for (int k = 0; k < nseg; ++k) M = fmaxf(M, grec[k * gstride + G * D + g]);
     float l = 0.f, acc = 0.f;
     for (int w = first; w <= last; ++w) {
       const float* rec = v.partials + (size_t)(w + bh) * v.record_floats;
+      const float sc = exp2f(rec[G * D + g] - M);
+      l = fmaf(rec[G * D + G + g], sc, l);
+      acc = fmaf(rec[e], sc, acc);
+    }
+    for (int k = 0; k < nseg; ++k) {
+      const float* rec = grec + k * gstride;
       const float sc = exp2f(rec[G * D + g] - M);
       l = fmaf(rec[G * D + G + g], sc, l);
       acc = fmaf(rec[e], sc, acc);

@@ -17,6 +17,7 @@ constexpr int kDecodeStages = 3;   // TMA ring depth per warp
 constexpr int kDecodeCtasPerSm = 1;
 constexpr int kMaxDecodeWarps = 4096;
 constexpr int kMaxCowJobs = 1024;
+constexpr int kMaxSegDepth = 16;   // grouped segments per beam (deeper shared levels use the per-beam path)
 
 // Control words at the start of the metadata buffer.
 enum Ctl : int {
@@ -27,6 +28,9 @@ enum Ctl : int {
   kCtlNextLineage = 4, // next lineage id to hand out
   kCtlFree = 5,        // number of free pages
   kCtlCowJobs = 6,     // copy-on-write jobs of the open step (rows copied by each layer's append)
+  kCtlSegCount = 7,    // shared-prefix segments found by the last rebuild
+  kCtlSegMembers = 8,  // (beam, depth) memberships handed out by the last rebuild
+  kCtlSegTiles = 9,    // 128-row query tiles over all segments
   kCtlWords = 32
 };
 
@@ -34,6 +38,9 @@ enum Ctl : int {
 struct MetaLayout {
   size_t ctl, tables, seq_len, active, gen, nsteps, mean, lineage, refcnt, free_bits;
   size_t plan, cow, partials, total;
+  // shared-prefix segments
+  size_t seg_cover, seg_nseg, seg_bstart, seg_bpage, seg_owner, seg_id, seg_i0, seg_len, seg_rep, seg_g,
+      seg_mem_off, seg_fill, seg_members, seg_tile_seg, seg_tile_t, grec;
   int words;            // free-bitmap words
   int partial_records;  // split-KV partial records
   int record_floats;    // floats per partial record: G*(D+2)
@@ -59,6 +66,25 @@ struct PoolView {
   unsigned* free_bits;
   int* plan;            // [2 modes][3][max_beams + 1]: offsets, chunk counts, start tokens
   int* cow;             // [kMaxCowJobs][3] (old page, new page, rows) of the open step's copy-on-writes
+  // Shared-prefix segments (rebuilt after seed, prune/branch and release):
+  int grouped;          // 1 when the grouped tensor-core path exists for this pool's dtype/shape
+  int group_min;        // segments need at least this many sharing beams
+  int* seg_cover;       // [max_beams] leading full pages of the beam covered by segments
+  int* seg_nseg;        // [max_beams] segments the beam belongs to (by depth)
+  int* seg_bstart;      // [max_beams][kMaxSegDepth] first table index of the beam's k-th segment
+  int* seg_bpage;       // [max_beams][kMaxSegDepth] page id at that index
+  unsigned long long* seg_owner;  // [num_pages] (rebuild gen << 32 | ~lowest beam) at segment-start pages
+  int* seg_id;          // [num_pages] segment id of a segment-start page
+  int* seg_i0;          // [segments] first table index
+  int* seg_len;         // [segments] pages
+  int* seg_rep;         // [segments] a member beam whose table lists the pages
+  int* seg_g;           // [segments] member beams
+  int* seg_mem_off;     // [segments] offset of its members
+  int* seg_fill;        // [segments] members written so far
+  int* seg_members;     // [memberships] beam * kMaxSegDepth + depth
+  int* seg_tile_seg;    // [tiles] segment of each 128-row query tile
+  int* seg_tile_t;      // [tiles] tile index within the segment
+  float* grec;          // [max_beams][kMaxSegDepth][Hkv] grouped partial records
   float* partials;
   int record_floats;
 };
@@ -147,6 +173,9 @@ struct gb_pool {
   int step_tokens;    // tokens reserved by the open step
   bool seeded;
   int group_min;
+  unsigned long long seg_gen = 0;           // segment rebuilds so far
+  alignas(64) unsigned char tmap[128];      // CUtensorMap over the KV pool (grouped path)
+  bool have_tmap = false;
   std::string last_error;
   unsigned long long launches = 0;          // kernels launched by this pool
   cudaEvent_t prof_start[GB_PROF_SLOTS] = {};  // caller-owned instrumentation events
@@ -170,6 +199,9 @@ cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, 
                           cudaStream_t s);
 cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* q, float scale, float* out,
                                cudaStream_t s);
+cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s);
+cudaError_t launch_grouped(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s);
+bool make_kv_tensor_map(gb_pool* pool);
 cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
                          float bias, const uint8_t* mask, float* score_out, const float* scores_in,
                          cudaStream_t s);

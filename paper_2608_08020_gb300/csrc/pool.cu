@@ -37,6 +37,23 @@ MetaLayout meta_layout(const gb_pool_config& c) {
   m.record_floats = G * (c.head_dim + 2);
   m.partial_records = kMaxDecodeWarps + (int)B * c.num_kv_heads;
   m.partials = take((size_t)m.partial_records * m.record_floats * sizeof(float));
+  const size_t BD = B * kMaxSegDepth;
+  m.seg_cover = take(B * sizeof(int));
+  m.seg_nseg = take(B * sizeof(int));
+  m.seg_bstart = take(BD * sizeof(int));
+  m.seg_bpage = take(BD * sizeof(int));
+  m.seg_owner = take((size_t)c.num_pages * sizeof(unsigned long long));
+  m.seg_id = take((size_t)c.num_pages * sizeof(int));
+  m.seg_i0 = take(BD * sizeof(int));
+  m.seg_len = take(BD * sizeof(int));
+  m.seg_rep = take(BD * sizeof(int));
+  m.seg_g = take(BD * sizeof(int));
+  m.seg_mem_off = take(BD * sizeof(int));
+  m.seg_fill = take(BD * sizeof(int));
+  m.seg_members = take(BD * sizeof(int));
+  m.seg_tile_seg = take(BD * sizeof(int));
+  m.seg_tile_t = take(BD * sizeof(int));
+  m.grec = take(BD * c.num_kv_heads * m.record_floats * sizeof(float));
   m.total = o;
   return m;
 }
@@ -447,8 +464,30 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   v.cow = reinterpret_cast<int*>(m + L.cow);
   v.partials = reinterpret_cast<float*>(m + L.partials);
   v.record_floats = L.record_floats;
+  v.seg_cover = reinterpret_cast<int*>(m + L.seg_cover);
+  v.seg_nseg = reinterpret_cast<int*>(m + L.seg_nseg);
+  v.seg_bstart = reinterpret_cast<int*>(m + L.seg_bstart);
+  v.seg_bpage = reinterpret_cast<int*>(m + L.seg_bpage);
+  v.seg_owner = reinterpret_cast<unsigned long long*>(m + L.seg_owner);
+  v.seg_id = reinterpret_cast<int*>(m + L.seg_id);
+  v.seg_i0 = reinterpret_cast<int*>(m + L.seg_i0);
+  v.seg_len = reinterpret_cast<int*>(m + L.seg_len);
+  v.seg_rep = reinterpret_cast<int*>(m + L.seg_rep);
+  v.seg_g = reinterpret_cast<int*>(m + L.seg_g);
+  v.seg_mem_off = reinterpret_cast<int*>(m + L.seg_mem_off);
+  v.seg_fill = reinterpret_cast<int*>(m + L.seg_fill);
+  v.seg_members = reinterpret_cast<int*>(m + L.seg_members);
+  v.seg_tile_seg = reinterpret_cast<int*>(m + L.seg_tile_seg);
+  v.seg_tile_t = reinterpret_cast<int*>(m + L.seg_tile_t);
+  v.grec = reinterpret_cast<float*>(m + L.grec);
+  v.group_min = p->group_min;
+  // The grouped tensor-core path needs bf16 K/V with D = 128 (kind::f16 MMAs, 128-byte rows).
+  v.grouped = (cfg->kv_dtype == GB_BF16 && cfg->head_dim == 128) ? 1 : 0;
+  if (v.grouped && !make_kv_tensor_map(p)) v.grouped = 0;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(m, 0, L.partials, s) != cudaSuccess) {
+  if (cudaMemsetAsync(m, 0, L.partials, s) != cudaSuccess ||
+      cudaMemsetAsync(m + L.seg_cover, 0, L.seg_owner - L.seg_cover, s) != cudaSuccess ||
+      cudaMemsetAsync(m + L.seg_owner, 0, (size_t)cfg->num_pages * sizeof(unsigned long long), s) != cudaSuccess) {
     delete p;
     return GB_ERR_CUDA;
   }
@@ -494,6 +533,7 @@ extern "C" gb_status gb_pool_seed(gb_pool* pool, int n_beams, int prompt_len, co
   st = check_launch(pool, "seed_write");
   if (st != GB_OK) return st;
   pool->seeded = true;
+  if (rebuild_segments(pool, s) != cudaSuccess) return check_launch(pool, "segments");
   return GB_OK;
 }
 
@@ -506,7 +546,7 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
     return fail(pool, GB_ERR_INVALID, "append: bad arguments");
   if (layer != pool->next_layer) return fail(pool, GB_ERR_STATE, "layers of a step must be called in order");
   if (layer == 0) {
-    k_step_begin<<<1, 1024, 0, s>>>(pool->view, n_tokens, nullptr);
+    k_step_begin<<<1, 1024, 0, s>>>(pool->view, n_tokens, pool->view.grouped ? pool->view.seg_cover : nullptr);
     pool->launches += 1;
     gb_status st = check_launch(pool, "step_begin");
     if (st != GB_OK) return st;
@@ -541,7 +581,10 @@ extern "C" gb_status gb_decode_attention(gb_pool* pool, int layer, const void* q
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   gb_status st = append_layer(pool, layer, 1, k_new_dev, v_new_dev, s);
   if (st != GB_OK) return st;
-  const int mode = 0;  // grouped coverage is applied when segments exist
+  // Mode 1: shared-prefix segments go through the grouped tensor-core kernel and the
+  // per-beam kernel reads only each beam's remainder; mode 0: every beam reads everything.
+  const int mode = (flags == GB_PATH_PER_BEAM || !pool->view.grouped) ? 0 : 1;
+  if (mode == 1 && launch_grouped(pool, layer, q_dev, scale, s) != cudaSuccess) return check_launch(pool, "grouped");
   if (launch_decode(pool, layer, q_dev, scale, out_dev, mode, s) != cudaSuccess)
     return check_launch(pool, "decode");
   return check_launch(pool, "decode");
@@ -554,7 +597,11 @@ extern "C" gb_status gb_release(gb_pool* pool, const int32_t* slots_dev, int n, 
   if (n == 0) return GB_OK;
   k_release<<<1, 1024, 0, reinterpret_cast<cudaStream_t>(stream)>>>(pool->view, slots_dev, n);
   pool->launches += 1;
-  return check_launch(pool, "release");
+  gb_status st = check_launch(pool, "release");
+  if (st != GB_OK) return st;
+  if (rebuild_segments(pool, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return check_launch(pool, "segments");
+  return GB_OK;
 }
 
 extern "C" gb_status gb_pool_status(gb_pool* pool, int* device_status, gb_stream_t stream) {

@@ -183,7 +183,10 @@ extern "C" gb_status gb_prune_branch(gb_pool* pool, int K, int fanout, int warmu
   if (K < 0 || fanout < 2) return fail(pool, GB_ERR_INVALID, "prune_branch: K >= 0 and fanout >= 2 required");
   if (!pool->seeded) return fail(pool, GB_ERR_STATE, "pool not seeded");
   if (pool->next_layer != 0) return fail(pool, GB_ERR_STATE, "prune_branch inside an open step");
-  launch_prune_branch(pool, K, fanout, warmup, eligible_dev, parent_out_dev, pruned_out_dev, lineage_out_dev,
-                      reinterpret_cast<cudaStream_t>(stream));
-  return check_launch(pool, "prune_branch");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  launch_prune_branch(pool, K, fanout, warmup, eligible_dev, parent_out_dev, pruned_out_dev, lineage_out_dev, s);
+  gb_status st = check_launch(pool, "prune_branch");
+  if (st != GB_OK) return st;
+  if (rebuild_segments(pool, s) != cudaSuccess) return check_launch(pool, "segments");
+  return GB_OK;
 }

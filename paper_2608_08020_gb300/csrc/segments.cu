@@ -1,0 +1,147 @@
+// Shared-prefix segments for the grouped attention path.
+//
+// A branched child shares every full page of its parent's prefix (Section 3.1,
+// after Eq. 3), so the beams that hold the page at table index i are exactly the
+// beams that also share every index before i.  Along one beam's table the number
+// of sharers (the page refcount) therefore never increases, and it changes exactly
+// where the set of sharers changes.  A segment is a maximal run of full pages of one
+// beam with a constant sharer set of at least `group_min` beams; every sharer of a
+// segment sees the same run at the same table indices.  The grouped kernel reads a
+// segment's pages once for all its sharers instead of once per beam.
+//
+// Rebuild (after seed, prune/branch and release; the set only changes there):
+//   1. scan:    one warp per beam walks its table, records the starts of its
+//               segments (up to kMaxSegDepth) and how many leading pages they cover,
+//               and marks each start page with the lowest beam that starts there;
+//   2. lead:    the lowest beam of each segment creates it (id, pages, member count);
+//   3. members: every member appends (beam, depth) to its segment's member list;
+//   4. tiles:   one CTA lays the segments' 128-row query tiles out as a flat list.
+// Segment ids and member order follow atomics, but each output row is computed
+// independently of its position, so results do not depend on that order.
+#include "internal.cuh"
+
+namespace gb {
+
+__global__ void k_seg_scan(PoolView v, unsigned long long gen) {
+  const int lane = threadIdx.x & 31;
+  const int b = (int)((blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    v.ctl[kCtlSegCount] = 0;
+    v.ctl[kCtlSegMembers] = 0;
+    v.ctl[kCtlSegTiles] = 0;
+  }
+  if (b >= v.max_beams) return;
+  int cover = 0, nseg = 0;
+  if (v.grouped && v.active[b]) {
+    const int nfull = v.seq_len[b] / v.P;
+    const int* tb = v.tables + (size_t)b * v.max_pages;
+    int prev_g = -1;
+    for (int i0 = 0; i0 < nfull; i0 += 32) {
+      const int i = i0 + lane;
+      int p = -1, g = 0;
+      if (i < nfull) {
+        p = tb[i];
+        g = (p >= 0 && p < v.num_pages) ? v.refcnt[p] : 0;
+      }
+      const unsigned low = __ballot_sync(0xffffffffu, i < nfull && g < v.group_min);
+      const int valid = min(32, nfull - i0);
+      const int lim = low ? min(valid, __ffs(low) - 1) : valid;  // positions still covered in this chunk
+      int gprev = __shfl_up_sync(0xffffffffu, g, 1);
+      if (lane == 0) gprev = prev_g;
+      unsigned starts = __ballot_sync(0xffffffffu, lane < lim && g != gprev);
+      bool stop = low != 0 || lim < 32;
+      while (starts) {
+        const int l = __ffs(starts) - 1;
+        starts &= starts - 1;
+        if (nseg == kMaxSegDepth) {  // deeper levels stay on the per-beam path
+          cover = i0 + l;
+          stop = true;
+          goto done;
+        }
+        const int pl = __shfl_sync(0xffffffffu, p, l);
+        if (lane == 0) {
+          v.seg_bstart[b * kMaxSegDepth + nseg] = i0 + l;
+          v.seg_bpage[b * kMaxSegDepth + nseg] = pl;
+          atomicMax(&v.seg_owner[pl], (gen << 32) | (unsigned long long)(0xffffffffu - (unsigned)b));
+        }
+        ++nseg;
+      }
+      cover = i0 + lim;
+      if (stop) break;
+      prev_g = __shfl_sync(0xffffffffu, g, 31);
+    }
+  }
+done:
+  if (lane == 0) {
+    v.seg_cover[b] = cover;
+    v.seg_nseg[b] = nseg;
+  }
+}
+
+__global__ void k_seg_lead(PoolView v, unsigned long long gen) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  const int b = idx / kMaxSegDepth, k = idx % kMaxSegDepth;
+  if (b >= v.max_beams || k >= v.seg_nseg[b]) return;
+  const int p0 = v.seg_bpage[b * kMaxSegDepth + k];
+  const unsigned long long ow = v.seg_owner[p0];
+  if ((ow >> 32) != gen || (0xffffffffu - (unsigned)(ow & 0xffffffffu)) != (unsigned)b) return;
+  const int id = atomicAdd(&v.ctl[kCtlSegCount], 1);
+  const int g = v.refcnt[p0];
+  const int off = atomicAdd(&v.ctl[kCtlSegMembers], g);
+  const int i0 = v.seg_bstart[b * kMaxSegDepth + k];
+  const int end = (k + 1 < v.seg_nseg[b]) ? v.seg_bstart[b * kMaxSegDepth + k + 1] : v.seg_cover[b];
+  v.seg_i0[id] = i0;
+  v.seg_len[id] = end - i0;
+  v.seg_rep[id] = b;
+  v.seg_g[id] = g;
+  v.seg_mem_off[id] = off;
+  v.seg_fill[id] = 0;
+  v.seg_id[p0] = id;
+}
+
+__global__ void k_seg_members(PoolView v) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  const int b = idx / kMaxSegDepth, k = idx % kMaxSegDepth;
+  if (b >= v.max_beams || k >= v.seg_nseg[b]) return;
+  const int id = v.seg_id[v.seg_bpage[b * kMaxSegDepth + k]];
+  const int slot = atomicAdd(&v.seg_fill[id], 1);
+  const int cap = v.max_beams * kMaxSegDepth;
+  if (slot < v.seg_g[id] && v.seg_mem_off[id] + slot < cap) v.seg_members[v.seg_mem_off[id] + slot] = idx;
+}
+
+// One CTA: flat list of 128-row query tiles (members * G rows per segment).
+__global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
+  __shared__ int tmp[33];
+  const int nseg = v.ctl[kCtlSegCount];
+  const int rows_per_tile = 128;
+  const int cap = v.max_beams * kMaxSegDepth;
+  int carry = 0;
+  for (int base = 0; base < nseg; base += blockDim.x) {
+    const int s = base + threadIdx.x;
+    const int tiles = s < nseg ? (v.seg_g[s] * v.G + rows_per_tile - 1) / rows_per_tile : 0;
+    int total;
+    const int off = carry + block_exclusive_scan(tiles, tmp, &total);
+    for (int t = 0; t < tiles && off + t < cap; ++t) {
+      v.seg_tile_seg[off + t] = s;
+      v.seg_tile_t[off + t] = t;
+    }
+    carry += total;
+  }
+  if (threadIdx.x == 0) v.ctl[kCtlSegTiles] = carry < cap ? carry : cap;
+}
+
+cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s) {
+  const PoolView& v = pool->view;
+  if (!v.grouped) return cudaSuccess;
+  const unsigned long long gen = ++pool->seg_gen;
+  const int warps_per_block = 8;
+  k_seg_scan<<<(v.max_beams + warps_per_block - 1) / warps_per_block, warps_per_block * 32, 0, s>>>(v, gen);
+  const int n = v.max_beams * kMaxSegDepth;
+  k_seg_lead<<<(n + 255) / 256, 256, 0, s>>>(v, gen);
+  k_seg_members<<<(n + 255) / 256, 256, 0, s>>>(v);
+  k_seg_tiles<<<1, 1024, 0, s>>>(v);
+  pool->launches += 4;
+  return cudaGetLastError();
+}
+
+}  // namespace gb
