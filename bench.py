@@ -45,6 +45,7 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", type=int, default=2, help="workload index 1..5 (default 2: the metric's config)")
     ap.add_argument("--flags", choices=["auto", "per_beam"], default="auto")
+    ap.add_argument("--group-min", type=int, default=0, help="beams a segment needs for the grouped path (0: 16)")
     ap.add_argument("--cpu-steps", type=int, default=6, help="steps of the oracle sample for cpu_baseline")
     ap.add_argument("--cpu-beams", type=int, default=16, help="beams per step in the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -220,7 +221,7 @@ def run_ours(args) -> None:
     W, K = args.warmup, args.steps
     S = W + 2 * K
 
-    g = GpuRun(wl, device_gen=True, device=str(dev), max_context=wl.context + S + 1)
+    g = GpuRun(wl, device_gen=True, device=str(dev), max_context=wl.context + S + 1, group_min_beams=args.group_min)
     t_build = time.perf_counter()
     g.build(upto=wl.context)
     torch.cuda.synchronize()
@@ -263,6 +264,7 @@ def run_ours(args) -> None:
         return evs
     n_dec = K * NL
     dec_a, dec_b = events(n_dec), events(n_dec)
+    gr_a, gr_b = events(n_dec), events(n_dec)
     pr_a, pr_b, pb_a, pb_b = events(K), events(K), events(K), events(K)
     torch.cuda.synchronize()
     launches0 = B.gb_pool_launch_count(pool.handle)
@@ -279,6 +281,7 @@ def run_ours(args) -> None:
         B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PROBE, pb_a[k], pb_b[k])
         for l in range(NL):
             B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_DECODE, dec_a[k * NL + l], dec_b[k * NL + l])
+            B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_GROUPED, gr_a[k * NL + l], gr_b[k * NL + l])
             pool.decode_attention(l, qs[i, l], ks[i, l], vs[i, l], wl.attn_scale, out[l], flags)
         pool.score_probe(hs[i], wl.hidden_dtype, g.w, wl.bias, None, g.scores)
         pool.prune_branch(wl.K, wl.fanout, wl.warmup, None, g.parent, g.pruned, g.lineage)
@@ -287,8 +290,9 @@ def run_ours(args) -> None:
     if world > 1:
         dist.barrier()
     clk = clocks.stop()
-    for which in (B.GB_PROF_DECODE, B.GB_PROF_PROBE, B.GB_PROF_PRUNE):
+    for which in (B.GB_PROF_DECODE, B.GB_PROF_PROBE, B.GB_PROF_PRUNE, B.GB_PROF_GROUPED):
         B.gb_pool_set_profile_events(pool.handle, which, None, None)
+    stats = B.gb_pool_read_step_stats(pool.handle, max_steps=K)  # one record per timed step (layer 0 opens it)
     launches = B.gb_pool_launch_count(pool.handle) - launches0
     elapsed_ms = t_start.elapsed_time(t_end)
     if world > 1:
@@ -302,17 +306,54 @@ def run_ours(args) -> None:
     if status != 0:
         raise RuntimeError(f"device status {status} after the timed steps: the measurement is invalid")
 
-    # Algorithmic bytes of one decode-kernel launch: every beam's K and V once, plus its queries.
-    kv_tok = 2 * Hkv * D * (2 if wl.kv_dtype == "bf16" else 4)
-    q_bytes = C * Hq * D * (2 if wl.kv_dtype == "bf16" else 4)
-    ctx_lens = [pos0 + k + 1 for k in range(K)]
-    alg_bytes = statistics.mean(C * L * kv_tok + q_bytes for L in ctx_lens)
+    gr_ms = [a.elapsed_time(b) for a, b in zip(gr_a, gr_b)]
+    grouped_on = flags != B.GB_PATH_PER_BEAM and wl.kv_dtype == "bf16" and D == 128
+
+    # Algorithmic work per launch, from the library's per-step records:
+    #   k_decode:  tokens it reads (all KV heads, K and V) + the queries;
+    #   k_grouped: K/V tiles it reads (once per 128-row query tile) and the useful flops
+    #              4 * D per (query row, token) for Q.K^T and P.V.
+    esz = 2 if wl.kv_dtype == "bf16" else 4
+    kv_tok = 2 * Hkv * D * esz
+    q_bytes = C * Hq * D * esz
+    assert len(stats) == K, (len(stats), K)
+    dec_tokens = [int(s[1] if grouped_on else s[0]) for s in stats]
+    dec_bytes = statistics.mean(t * kv_tok + q_bytes for t in dec_tokens)
+    eff_bytes = statistics.mean(int(s[0]) * kv_tok + q_bytes for s in stats)   # as if every beam read everything
+    gr_bytes = statistics.mean(Hkv * int(s[3]) * 2 * D * esz for s in stats) if grouped_on else 0.0
+    gr_flops = statistics.mean(Hkv * int(s[2]) * 4 * D for s in stats) if grouped_on else 0.0
     dec_avg_s = statistics.mean(dec_ms) / 1e3
-    achieved = alg_bytes / dec_avg_s / 1e9
+    gr_avg_s = statistics.mean(gr_ms) / 1e3 if grouped_on else 0.0
+    achieved = dec_bytes / dec_avg_s / 1e9
     peaks = measured_peaks()
     peak = peaks.get("hbm_gbs")
     peak_src = "measured" if peak else "fallback"
     peak = peak or 6800.0
+    tpeak = peaks.get("bf16_tflops_sustained") or peaks.get("bf16_tflops")
+    tpeak_src = "measured sustained" if tpeak else "fallback"
+    tpeak = tpeak or 1700.0
+    kernels = {"k_decode": {"us": dec_avg_s * 1e6, "bytes": dec_bytes, "gbps": achieved, "frac_hbm": achieved / peak}}
+    if grouped_on and gr_avg_s > 0:
+        kernels["k_grouped"] = {"us": gr_avg_s * 1e6, "bytes": gr_bytes, "gbps": gr_bytes / gr_avg_s / 1e9,
+                                "frac_hbm": gr_bytes / gr_avg_s / 1e9 / peak, "flops": gr_flops,
+                                "tflops": gr_flops / gr_avg_s / 1e12, "frac_tensor": gr_flops / gr_avg_s / 1e12 / tpeak,
+                                "segments": statistics.mean(int(s[4]) for s in stats),
+                                "tiles": statistics.mean(int(s[5]) for s in stats)}
+    dominant = "k_grouped" if "k_grouped" in kernels and gr_avg_s > dec_avg_s else "k_decode"
+    if dominant == "k_decode":
+        roofline = {"bound": "hbm", "kernel": "k_decode (split-KV decode)", "achieved": achieved, "peak": peak,
+                    "unit": "GB/s", "frac": achieved / peak, "traffic": None, "bytes_per_launch": dec_bytes,
+                    "peak_source": f"{peak_src} hbm_gbs"}
+    else:
+        kg = kernels["k_grouped"]
+        if kg["frac_tensor"] >= kg["frac_hbm"]:
+            roofline = {"bound": "tensor", "kernel": "k_grouped (tcgen05 shared-prefix)", "achieved": kg["tflops"],
+                        "peak": tpeak, "unit": "TFLOP/s", "frac": kg["frac_tensor"], "traffic": None,
+                        "flops_per_launch": gr_flops, "peak_source": f"{tpeak_src} bf16_tflops"}
+        else:
+            roofline = {"bound": "hbm", "kernel": "k_grouped (tcgen05 shared-prefix)", "achieved": kg["gbps"],
+                        "peak": peak, "unit": "GB/s", "frac": kg["frac_hbm"], "traffic": None,
+                        "bytes_per_launch": gr_bytes, "peak_source": f"{peak_src} hbm_gbs"}
 
     value = world * C * K / (elapsed_ms / 1e3)
     ms_per_step = elapsed_ms / K
@@ -376,13 +417,15 @@ def run_ours(args) -> None:
                        "path": args.flags, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "l2": f"inputs larger than L2: {C * pos0 * kv_tok / 2**30:.2f} GiB of KV read per step",
                        "tree_build_s": round(t_build, 2)},
-            "attention_tbps": achieved / 1e3,
+            "attention_us": (dec_avg_s + gr_avg_s) * 1e6,
+            "attention_tbps": eff_bytes / (dec_avg_s + gr_avg_s) / 1e12,
+            "attention_tbps_note": "every beam's whole context (K and V of all KV heads) per attention time",
             "decode_kernel_us": dec_avg_s * 1e6,
+            "grouped_kernel_us": gr_avg_s * 1e6,
             "probe_us": probe_us,
             "prune_branch_us": prune_us,
-            "roofline": {"bound": "hbm", "kernel": "k_decode (split-KV decode)", "achieved": achieved, "peak": peak,
-                         "unit": "GB/s", "frac": achieved / peak, "traffic": None,
-                         "bytes_per_launch": alg_bytes, "peak_source": f"{peak_src} hbm_gbs"},
+            "kernels": kernels,
+            "roofline": roofline,
             "e2e": e2e,
             "gpu_launches": int(launches),
             "clocks": clk,

@@ -86,6 +86,8 @@ typedef struct {
   uint32_t* lineage;   /* [max_beams] unique id of the beam now in the slot */
   int32_t* refcnt;     /* [num_pages] active slots referencing each page */
   uint32_t* free_bits; /* [ceil(num_pages/32)] bit p%32 of word p/32 set when page p is free */
+  int32_t* seg_cover;  /* [max_beams] leading full pages read by the grouped path (0 without it) */
+  int32_t* seg_nseg;   /* [max_beams] shared-prefix segments covering them */
 } gb_pool_state;
 
 /*
@@ -240,6 +242,18 @@ gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_strea
 #define GB_PROF_GROUPED 3
 #define GB_PROF_SLOTS 4
 gb_status gb_pool_set_profile_events(gb_pool* pool, int which, void* start_event, void* stop_event);
+
+/*
+ * Work accounting of the most recent decode/append steps (not part of the method).
+ * Synchronises `stream` and copies up to max_steps records, oldest first, into
+ * out[n][8] (host): [0] tokens per KV head the per-beam path reads when every
+ * beam reads its whole context, [1] the same with shared-prefix segments taken
+ * by the grouped path, [2] sum over segments of (query rows of one KV head) x
+ * tokens, [3] sum over segments of (128-row tiles) x tokens, [4] segments,
+ * [5] 128-row tiles, [6] tokens appended by the step, [7] step index.
+ * *n_out receives the number of records (at most the last 4096 steps are kept).
+ */
+gb_status gb_pool_read_step_stats(gb_pool* pool, int32_t* out, int max_steps, int* n_out, gb_stream_t stream);
 
 /* Number of kernels this pool has launched since gb_pool_init (host-side count). */
 gb_status gb_pool_launch_count(gb_pool* pool, uint64_t* count);

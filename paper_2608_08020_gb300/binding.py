@@ -27,7 +27,7 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
            "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
-           "gb_paged_decode_noalloc", "gb_last_error"]
+           "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
 
 
@@ -41,7 +41,8 @@ class GbPoolConfig(ctypes.Structure):
 class GbPoolState(ctypes.Structure):
     _fields_ = [("tables", ctypes.c_void_p), ("seq_len", ctypes.c_void_p), ("active", ctypes.c_void_p),
                 ("gen", ctypes.c_void_p), ("nsteps", ctypes.c_void_p), ("mean", ctypes.c_void_p),
-                ("lineage", ctypes.c_void_p), ("refcnt", ctypes.c_void_p), ("free_bits", ctypes.c_void_p)]
+                ("lineage", ctypes.c_void_p), ("refcnt", ctypes.c_void_p), ("free_bits", ctypes.c_void_p),
+                ("seg_cover", ctypes.c_void_p), ("seg_nseg", ctypes.c_void_p)]
 
 
 class GbPagedDecodeArgs(ctypes.Structure):
@@ -88,6 +89,7 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_pool_set_profile_events": [V, I, V, V],
         "gb_pool_launch_count": [V, P],
         "gb_paged_decode_noalloc": [P, V],
+        "gb_pool_read_step_stats": [V, P, I, P, V],
         "gb_last_error": [V],
     }
     for name, args in sig.items():
@@ -207,6 +209,20 @@ def gb_pool_set_profile_events(pool: int, which: int, start_event=None, stop_eve
         return e.cuda_event
     _check(pool, load().gb_pool_set_profile_events(pool, which, ev(start_event), ev(stop_event)),
            "gb_pool_set_profile_events")
+
+
+STEP_STATS_FIELDS = ("tokens_per_beam_path", "tokens_with_grouped", "seg_rowtok", "seg_tiletok", "segments",
+                     "tiles", "appended", "step")
+
+
+def gb_pool_read_step_stats(pool: int, max_steps: int = 4096, stream=None):
+    """Work records of the last steps: an int32 array [n][8] (see include/gambit.h)."""
+    import numpy as np
+    out = np.zeros((max_steps, 8), dtype=np.int32)
+    n = ctypes.c_int()
+    _check(pool, load().gb_pool_read_step_stats(pool, out.ctypes.data, max_steps, ctypes.byref(n),
+                                                stream_handle(stream)), "gb_pool_read_step_stats")
+    return out[:n.value]
 
 
 def gb_pool_launch_count(pool: int) -> int:

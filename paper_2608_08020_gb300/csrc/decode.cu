@@ -406,7 +406,7 @@ __global__ void k_combine(PoolView v, int mode, int W, float* __restrict__ out) 
   float* ob = out + ((size_t)b * v.Hq + (size_t)h * G) * D;
   const bool ok = v.ctl[kCtlStepOk] != 0 && v.active[b] != 0;
   const int n = ok ? plan_n(v, mode)[b] : 0;
-  const int nseg = (ok && mode == 1 && v.grouped) ? v.seg_nseg[b] : 0;
+  const int nseg = (ok && mode == 1 && v.grouped) ? v.seg_nrec[b] : 0;  // grouped records of the beam
   if (n == 0 && nseg == 0) {
     for (int e = threadIdx.x; e < G * D; e += blockDim.x) ob[e] = 0.f;
     return;
@@ -415,7 +415,7 @@ __global__ void k_combine(PoolView v, int mode, int W, float* __restrict__ out) 
   const int c = Tot > 0 ? (Tot + W - 1) / W : 1;
   const int off = plan_off(v, mode)[b] + h * n;
   const int first = off / c, last = n > 0 ? (off + n - 1) / c : first - 1;
-  const float* grec = v.grec + ((size_t)b * kMaxSegDepth * v.Hkv + h) * v.record_floats;
+  const float* grec = v.grec + ((size_t)b * kMaxSegRecords * v.Hkv + h) * v.record_floats;
   const size_t gstride = (size_t)v.Hkv * v.record_floats;
   for (int e = threadIdx.x; e < G * D; e += blockDim.x) {
     const int g = e / D;

@@ -33,7 +33,7 @@ namespace {
 
 constexpr int kRows = 128;     // query rows per tile (MMA M)
 constexpr int kTok = 64;       // tokens per K/V tile (MMA N of Q.K^T, K of P.V)
-constexpr int kStages = 2;
+constexpr int kStages = 4;
 constexpr int kThreads = 128;
 constexpr uint32_t kTmemCols = 256;  // S: columns [0, 64), O: [128, 256)
 
@@ -162,16 +162,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t loads_issued = 0, loads_used = 0, s_done = 0, pv_done = 0;
   bool timed_out = false;
 
-  auto issue_tile = [&](int seg_i0, int rep, int h, int Ts, int j, uint32_t stage) {
+  auto issue_tile = [&](int seg_i0, int tok_base, int rep, int h, int Ts, int j, uint32_t stage) {
     // Tokens [64j, 64j+64) of the segment: four 16-token chunks, K and V, two 64-dim halves.
     const uint32_t bar = bfull0 + 8 * stage;
     mbar_arrive_expect_tx(bar, kStage);
     const uint32_t dst0 = sbase + kKV + stage * kStage;
 #pragma unroll
     for (int c = 0; c < 4; ++c) {
-      const int tk = j * kTok + c * 16;
+      const int tk = tok_base + j * kTok + c * 16;  // token within the segment
       long long yk = total_rows, yv = total_rows;  // out of bounds: zero fill
-      if (tk < Ts) {
+      if (j * kTok + c * 16 < Ts) {
         int page = v.tables[(size_t)rep * v.max_pages + seg_i0 + tk / v.P];
         if (page < 0 || page >= v.num_pages) {
           set_status(v.ctl, GB_ERR_INVALID);
@@ -191,9 +191,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   for (long long u = blockIdx.x; u < units && !timed_out; u += gridDim.x) {
     const int tq = (int)(u / v.Hkv), h = (int)(u % v.Hkv);
-    const int s = v.seg_tile_seg[tq], t = v.seg_tile_t[tq];
+    const int s = v.seg_tile_seg[tq], t = v.seg_tile_t[tq], sp = v.seg_tile_split[tq];
+    const int split = v.ctl[kCtlSegSplit];
+    const int tok_base = sp * split;
     const int seg_i0 = v.seg_i0[s], rep = v.seg_rep[s], g = v.seg_g[s], moff = v.seg_mem_off[s];
-    const int Ts = v.seg_len[s] * v.P;
+    const int Ts = min(v.seg_len[s] * v.P - tok_base, split);  // tokens of this split
     const int ntok = (Ts + kTok - 1) / kTok;
     constexpr int members_per_tile = kRows / G;
 
@@ -217,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
 
     if (tid == 0) {
-      for (int j = 0; j < kStages && j < ntok; ++j) issue_tile(seg_i0, rep, h, Ts, j, (loads_issued + j) % kStages);
+      for (int j = 0; j < kStages && j < ntok; ++j) issue_tile(seg_i0, tok_base, rep, h, Ts, j, (loads_issued + j) % kStages);
     }
     uint32_t issued_here = ntok < kStages ? ntok : kStages;
 
@@ -268,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++pv_done;
         tc_fence_after();
         if (tid == 0 && j - 1 + kStages < ntok) {
-          issue_tile(seg_i0, rep, h, Ts, j - 1 + kStages, (gj - 1) % kStages);
+          issue_tile(seg_i0, tok_base, rep, h, Ts, j - 1 + kStages, (gj - 1) % kStages);
           ++issued_here;
         }
       }
@@ -333,9 +335,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     {
       const int r = tid;
       const int m = t * members_per_tile + r / G, gg = r % G;
-      const bool has = m < g;
-      const int bk = has ? v.seg_members[moff + m] : 0;
-      float* rec = v.grec + ((size_t)bk * v.Hkv + h) * v.record_floats;
+      const int bk = m < g ? v.seg_members[moff + m] : 0;
+      const int b = bk / kMaxSegDepth;
+      const int r_idx = v.seg_rec_off[bk] + sp;
+      const bool has = m < g && r_idx < kMaxSegRecords;
+      float* rec = v.grec + (((size_t)b * kMaxSegRecords + r_idx) * v.Hkv + h) * v.record_floats;
 #pragma unroll 1
       for (int c0 = 0; c0 < 128; c0 += 32) {  // warp-collective loads: every lane takes part
         float o[32];

@@ -17,7 +17,10 @@ constexpr int kDecodeStages = 3;   // TMA ring depth per warp
 constexpr int kDecodeCtasPerSm = 1;
 constexpr int kMaxDecodeWarps = 4096;
 constexpr int kMaxCowJobs = 1024;
-constexpr int kMaxSegDepth = 16;   // grouped segments per beam (deeper shared levels use the per-beam path)
+constexpr int kMaxSegDepth = 16;
+constexpr int kMaxSegRecords = 48;  // grouped partial records per beam (segments x token splits)
+constexpr int kStatsRing = 4096;   // steps kept in the step-stats ring
+constexpr int kStatsWords = 8;   // grouped segments per beam (deeper shared levels use the per-beam path)
 
 // Control words at the start of the metadata buffer.
 enum Ctl : int {
@@ -31,16 +34,21 @@ enum Ctl : int {
   kCtlSegCount = 7,    // shared-prefix segments found by the last rebuild
   kCtlSegMembers = 8,  // (beam, depth) memberships handed out by the last rebuild
   kCtlSegTiles = 9,    // 128-row query tiles over all segments
+  kCtlSegRowTok = 10,  // sum over segments of (query rows of one KV head) x tokens
+  kCtlSegTileTok = 11, // sum over segments of (128-row tiles) x tokens
+  kCtlSteps = 12,      // steps opened so far (index into the step-stats ring)
+  kCtlSegSplit = 13,   // tokens per grouped work unit (segments are split along tokens)
   kCtlWords = 32
 };
 
 // Byte offsets of the metadata regions.
 struct MetaLayout {
   size_t ctl, tables, seq_len, active, gen, nsteps, mean, lineage, refcnt, free_bits;
-  size_t plan, cow, partials, total;
+  size_t plan, cow, partials, total, stats;
   // shared-prefix segments
   size_t seg_cover, seg_nseg, seg_bstart, seg_bpage, seg_owner, seg_id, seg_i0, seg_len, seg_rep, seg_g,
-      seg_mem_off, seg_fill, seg_members, seg_tile_seg, seg_tile_t, grec;
+      seg_mem_off, seg_fill, seg_members, seg_tile_seg, seg_tile_t, grec, seg_bid, seg_rec_off, seg_nrec,
+      seg_splits, seg_tile_split;
   int words;            // free-bitmap words
   int partial_records;  // split-KV partial records
   int record_floats;    // floats per partial record: G*(D+2)
@@ -84,7 +92,14 @@ struct PoolView {
   int* seg_members;     // [memberships] beam * kMaxSegDepth + depth
   int* seg_tile_seg;    // [tiles] segment of each 128-row query tile
   int* seg_tile_t;      // [tiles] tile index within the segment
+  int* seg_tile_split;  // [tiles] token split of the unit
+  int* seg_splits;      // [segments] token splits of the segment
+  int* seg_bid;         // [max_beams][kMaxSegDepth] segment id of the beam's k-th segment
+  int* seg_rec_off;     // [max_beams][kMaxSegDepth] first grouped record of that segment
+  int* seg_nrec;        // [max_beams] grouped records of the beam
+  int num_sms;          // multiprocessors (sizes the grouped work split)
   float* grec;          // [max_beams][kMaxSegDepth][Hkv] grouped partial records
+  int* stats;           // [kStatsRing][kStatsWords] work of recent steps (see gb_pool_read_step_stats)
   float* partials;
   int record_floats;
 };

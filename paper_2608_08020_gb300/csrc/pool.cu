@@ -8,6 +8,7 @@
 // the order is exactly that sequential rule.
 #include <algorithm>
 #include <cstring>
+#include <vector>
 
 #include "internal.cuh"
 
@@ -51,9 +52,15 @@ MetaLayout meta_layout(const gb_pool_config& c) {
   m.seg_mem_off = take(BD * sizeof(int));
   m.seg_fill = take(BD * sizeof(int));
   m.seg_members = take(BD * sizeof(int));
-  m.seg_tile_seg = take(BD * sizeof(int));
-  m.seg_tile_t = take(BD * sizeof(int));
-  m.grec = take(BD * c.num_kv_heads * m.record_floats * sizeof(float));
+  m.seg_tile_seg = take(B * kMaxSegRecords * sizeof(int));  // work entries <= records
+  m.seg_tile_t = take(B * kMaxSegRecords * sizeof(int));
+  m.grec = take(B * kMaxSegRecords * c.num_kv_heads * m.record_floats * sizeof(float));
+  m.seg_bid = take(BD * sizeof(int));
+  m.seg_rec_off = take(BD * sizeof(int));
+  m.seg_nrec = take(B * sizeof(int));
+  m.seg_splits = take(BD * sizeof(int));
+  m.seg_tile_split = take(B * kMaxSegRecords * sizeof(int));
+  m.stats = take((size_t)kStatsRing * kStatsWords * sizeof(int));
   m.total = o;
   return m;
 }
@@ -204,6 +211,7 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
   __shared__ int s_alloc[kMaxBeams];
   __shared__ int s_tail[kMaxBeams];
   __shared__ int s_ncow;
+  __shared__ int s_tok[2];
   const int b = threadIdx.x;
   const bool act = b < v.max_beams && v.active[b] != 0;
   const int L = act ? v.seq_len[b] : 0;
@@ -295,6 +303,24 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
       plan_start(v, mode)[b] = start;
     }
     if (b == 0) plan_off(v, mode)[v.max_beams] = total;
+    int tok_total;
+    block_exclusive_scan(act ? Lnew - start : 0, tmp, &tok_total);
+    if (b == 0) s_tok[mode] = tok_total;
+  }
+  if (b == 0) {
+    // Work of this step: tokens each path reads per KV head, and the segment work of the
+    // grouped path (valid until the next rebuild).
+    const int step = v.ctl[kCtlSteps];
+    int* e = v.stats + (size_t)(step % kStatsRing) * kStatsWords;
+    e[0] = s_tok[0];
+    e[1] = s_tok[1];
+    e[2] = v.grouped ? v.ctl[kCtlSegRowTok] : 0;
+    e[3] = v.grouped ? v.ctl[kCtlSegTileTok] : 0;
+    e[4] = v.grouped ? v.ctl[kCtlSegCount] : 0;
+    e[5] = v.grouped ? v.ctl[kCtlSegTiles] : 0;
+    e[6] = n_tokens;
+    e[7] = step;
+    v.ctl[kCtlSteps] = step + 1;
   }
   if (b == 0) v.ctl[kCtlStepOk] = 1;
 }
@@ -480,6 +506,13 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   v.seg_tile_seg = reinterpret_cast<int*>(m + L.seg_tile_seg);
   v.seg_tile_t = reinterpret_cast<int*>(m + L.seg_tile_t);
   v.grec = reinterpret_cast<float*>(m + L.grec);
+  v.seg_bid = reinterpret_cast<int*>(m + L.seg_bid);
+  v.seg_rec_off = reinterpret_cast<int*>(m + L.seg_rec_off);
+  v.seg_nrec = reinterpret_cast<int*>(m + L.seg_nrec);
+  v.seg_splits = reinterpret_cast<int*>(m + L.seg_splits);
+  v.seg_tile_split = reinterpret_cast<int*>(m + L.seg_tile_split);
+  v.num_sms = p->num_sms;
+  v.stats = reinterpret_cast<int*>(m + L.stats);
   v.group_min = p->group_min;
   // The grouped tensor-core path needs bf16 K/V with D = 128 (kind::f16 MMAs, 128-byte rows).
   v.grouped = (cfg->kv_dtype == GB_BF16 && cfg->head_dim == 128) ? 1 : 0;
@@ -622,6 +655,27 @@ extern "C" gb_status gb_pool_set_profile_events(gb_pool* pool, int which, void* 
   return GB_OK;
 }
 
+extern "C" gb_status gb_pool_read_step_stats(gb_pool* pool, int32_t* out, int max_steps, int* n_out,
+                                             gb_stream_t stream) {
+  if (!pool || !out || !n_out || max_steps < 0) return GB_ERR_INVALID;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  std::vector<int> ring((size_t)kStatsRing * kStatsWords);
+  int steps = 0;
+  if (cudaMemcpyAsync(&steps, pool->view.ctl + kCtlSteps, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaMemcpyAsync(ring.data(), pool->view.stats, ring.size() * sizeof(int), cudaMemcpyDeviceToHost, s) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return check_launch(pool, "read_step_stats");
+  const int n = std::min({max_steps, steps, kStatsRing});
+  for (int i = 0; i < n; ++i) {
+    const int step = steps - n + i;
+    std::memcpy(out + (size_t)i * kStatsWords, ring.data() + (size_t)(step % kStatsRing) * kStatsWords,
+                kStatsWords * sizeof(int));
+  }
+  *n_out = n;
+  return GB_OK;
+}
+
 extern "C" gb_status gb_pool_launch_count(gb_pool* pool, uint64_t* count) {
   if (!pool || !count) return GB_ERR_INVALID;
   *count = pool->launches;
@@ -650,6 +704,8 @@ extern "C" gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* st, 
       {st->lineage, v.lineage, B * sizeof(unsigned)},
       {st->refcnt, v.refcnt, (size_t)v.num_pages * sizeof(int)},
       {st->free_bits, v.free_bits, (size_t)v.words * sizeof(unsigned)},
+      {st->seg_cover, v.seg_cover, B * sizeof(int)},
+      {st->seg_nseg, v.seg_nseg, B * sizeof(int)},
   };
   for (const Copy& c : copies) {
     if (!c.dst) continue;

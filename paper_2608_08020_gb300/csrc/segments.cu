@@ -104,28 +104,76 @@ __global__ void k_seg_members(PoolView v) {
   const int b = idx / kMaxSegDepth, k = idx % kMaxSegDepth;
   if (b >= v.max_beams || k >= v.seg_nseg[b]) return;
   const int id = v.seg_id[v.seg_bpage[b * kMaxSegDepth + k]];
+  v.seg_bid[idx] = id;
   const int slot = atomicAdd(&v.seg_fill[id], 1);
   const int cap = v.max_beams * kMaxSegDepth;
   if (slot < v.seg_g[id] && v.seg_mem_off[id] + slot < cap) v.seg_members[v.seg_mem_off[id] + slot] = idx;
 }
 
-// One CTA: flat list of 128-row query tiles (members * G rows per segment).
+// One CTA: the grouped work list.  Each segment has ceil(g*G/128) query tiles; each
+// tile is split along the segment's tokens into pieces of `split` tokens so that the
+// list has about two units per multiprocessor (and no beam needs more than
+// kMaxSegRecords partial records).  Entries are (segment, tile, split); every beam
+// gets the offsets of its records (one per split of each of its segments).
 __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
   __shared__ int tmp[33];
+  __shared__ int s_split;
   const int nseg = v.ctl[kCtlSegCount];
   const int rows_per_tile = 128;
-  const int cap = v.max_beams * kMaxSegDepth;
+  const int cap = v.max_beams * kMaxSegRecords;
+  int rowtok = 0, tiletok = 0;
+  for (int base = 0; base < nseg; base += blockDim.x) {
+    const int s = base + threadIdx.x;
+    const int tiles = s < nseg ? (v.seg_g[s] * v.G + rows_per_tile - 1) / rows_per_tile : 0;
+    const int toks = s < nseg ? v.seg_len[s] * v.P : 0;
+    int t1, t2;
+    block_exclusive_scan(s < nseg ? v.seg_g[s] * v.G * toks : 0, tmp, &t1);
+    block_exclusive_scan(tiles * toks, tmp, &t2);
+    rowtok += t1;
+    tiletok += t2;
+  }
+  if (threadIdx.x == 0) {
+    const long long work = (long long)tiletok * v.Hkv;              // tile-tokens over all heads
+    const long long target_units = 2LL * (v.num_sms > 0 ? v.num_sms : 1);
+    int split = (int)(((work + target_units - 1) / target_units + 63) / 64 * 64);
+    const int max_tokens = v.max_pages * v.P;
+    const int min_split = ((max_tokens + (kMaxSegRecords - kMaxSegDepth) - 1) / (kMaxSegRecords - kMaxSegDepth) + 63) /
+                          64 * 64;
+    split = max(split, max(128, min_split));
+    s_split = split;
+    v.ctl[kCtlSegSplit] = split;
+    v.ctl[kCtlSegRowTok] = rowtok;
+    v.ctl[kCtlSegTileTok] = tiletok;
+  }
+  __syncthreads();
+  const int split = s_split;
   int carry = 0;
   for (int base = 0; base < nseg; base += blockDim.x) {
     const int s = base + threadIdx.x;
     const int tiles = s < nseg ? (v.seg_g[s] * v.G + rows_per_tile - 1) / rows_per_tile : 0;
+    const int splits = s < nseg ? (v.seg_len[s] * v.P + split - 1) / split : 0;
+    if (s < nseg) v.seg_splits[s] = splits;
     int total;
-    const int off = carry + block_exclusive_scan(tiles, tmp, &total);
-    for (int t = 0; t < tiles && off + t < cap; ++t) {
-      v.seg_tile_seg[off + t] = s;
-      v.seg_tile_t[off + t] = t;
-    }
+    const int off = carry + block_exclusive_scan(tiles * splits, tmp, &total);
+    for (int t = 0; t < tiles; ++t)
+      for (int sp = 0; sp < splits; ++sp) {
+        const int e = off + t * splits + sp;
+        if (e < cap) {
+          v.seg_tile_seg[e] = s;
+          v.seg_tile_t[e] = t;
+          v.seg_tile_split[e] = sp;
+        }
+      }
     carry += total;
+  }
+  __syncthreads();
+  for (int b = threadIdx.x; b < v.max_beams; b += blockDim.x) {
+    int off = 0;
+    for (int k = 0; k < v.seg_nseg[b]; ++k) {
+      v.seg_rec_off[b * kMaxSegDepth + k] = off;
+      off += v.seg_splits[v.seg_bid[b * kMaxSegDepth + k]];
+    }
+    v.seg_nrec[b] = off < kMaxSegRecords ? off : kMaxSegRecords;
   }
   if (threadIdx.x == 0) v.ctl[kCtlSegTiles] = carry < cap ? carry : cap;
 }

@@ -87,8 +87,10 @@ class BeamPool:
             "active": np.zeros(C, np.int32), "gen": np.zeros(C, np.int32), "nsteps": np.zeros(C, np.int32),
             "mean": np.zeros(C, np.float32), "lineage": np.zeros(C, np.uint32),
             "refcnt": np.zeros(NP, np.int32), "free_bits": np.zeros((NP + 31) // 32, np.uint32),
+            "seg_cover": np.zeros(C, np.int32), "seg_nseg": np.zeros(C, np.int32),
         }
         st = B.GbPoolState(*[out[k].ctypes.data for k in ("tables", "seq_len", "active", "gen", "nsteps", "mean",
-                                                         "lineage", "refcnt", "free_bits")])
+                                                         "lineage", "refcnt", "free_bits", "seg_cover",
+                                                         "seg_nseg")])
         B.gb_pool_read_state(self.handle, st, stream)
         return out

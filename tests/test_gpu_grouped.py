@@ -7,6 +7,7 @@ import dataclasses
 import numpy as np
 import pytest
 
+from oracle.segments import segments
 from oracle.trajectory import OracleRun
 from paper_2608_08020_gb300 import binding as B
 from tests.parity import assert_close, assert_pool_equal
@@ -28,7 +29,13 @@ def test_grouped_matches_oracle(cuda, beams, group_min, prompt, context, interva
     o = OracleRun(wl, literal_kv=False)
     g.build(upto=context - 3)
     o.build(upto=context - 3)
-    assert_pool_equal(g.pool.read_state(), o.pool, wl.page_size, means="tol", dtype="bf16")
+    st = g.pool.read_state()
+    assert_pool_equal(st, o.pool, wl.page_size, means="tol", dtype="bf16")
+    cover, nseg, _ = segments(o.pool, group_min)
+    act = o.pool.active
+    assert np.array_equal(st["seg_cover"][act], cover[act]), (st["seg_cover"][act], cover[act])
+    assert np.array_equal(st["seg_nseg"][act], nseg[act])
+    assert cover.sum() > 0 and nseg.max() >= 1, "the grouped path must cover something here"
     for step in range(3):
         out = g.decode_step(B.GB_PATH_AUTO).cpu().numpy()
         ref = o.decode_step()
