@@ -1,15 +1,20 @@
 """Benchmark of the beam-decode hot path of thought-level beam search on GB300.
 
-One step = one pass of the whole hot path over the beam population:
-  decode attention of every active beam (page reservation + KV append +
-  split-KV attention + combine), the scorer probe with the running-mean
-  update, and one tournament round (rank, prune, fork block tables, free).
+The method's schedule: every decode step appends one token to every active
+beam and attends over its context (page reservation + KV append + grouped
+shared-prefix attention + per-beam split-KV attention + combine); every
+Delta tokens the probe scores every beam and one tournament round prunes and
+branches (rank, fork block tables, free pages, rebuild shared-prefix
+segments).  The timed window is K decode steps and contains the rounds that
+fall in it (by default one round: K = Delta), so every row of the hot path
+runs in it and the beam tree is the one the schedule produces.
 
 Default workload: the Qwen3-8B-shaped single layer (64 beams, 32/8 heads,
-head dim 128, bf16 KV, 16-token pages), its beam tree built by real rounds
-(prune/branch every 512 tokens, keep 50%, branch x2) up to 4096 tokens of
-context; timing starts there.  Inputs are seeded synthetic data generated
-on the device before the timed region.  The KV read per step (1 GiB) is far
+head dim 128, bf16 KV, 16-token pages), beam tree built by real rounds
+(prune/branch every 512 tokens, keep 50%, branch x2) up to 4096 tokens;
+the timed window runs from 4096 to 4608 tokens with the round at 4608.
+Inputs are seeded synthetic data generated on the device before the timed
+region.  The KV a step attends over (about 1 GiB as per-beam reads) is far
 larger than L2, so no flush is needed between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--config I]
@@ -40,8 +45,8 @@ if ROOT not in sys.path:
 def parse_args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=400)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=0, help="timed decode steps (0: one tournament interval)")
+    ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", type=int, default=2, help="workload index 1..5 (default 2: the metric's config)")
     ap.add_argument("--flags", choices=["auto", "per_beam"], default="auto")
@@ -112,6 +117,22 @@ def gpu_id_for_smi(local: int) -> str:
     except Exception:
         vis = os.environ.get("CUDA_VISIBLE_DEVICES")
         return vis.split(",")[local] if vis else str(local)
+
+
+def captured_traffic(kernel: str, workload: str, path: str):
+    """DRAM bytes per launch from the committed ncu capture, if it is of this kernel source and workload."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f).get(kernel)
+        if not rec or rec["workload"] != workload or rec["path"] != path:
+            return None
+        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
+                return None
+        return rec["dram_bytes_per_launch"]
+    except (OSError, KeyError, ValueError):
+        return None
 
 
 def measured_peaks() -> dict:
@@ -218,22 +239,30 @@ def run_ours(args) -> None:
     dev = torch.device("cuda", local)
     wl = dataclasses.replace(BY_INDEX[args.config - 1], seed=BY_INDEX[args.config - 1].seed + rank)
     flags = B.GB_PATH_AUTO if args.flags == "auto" else B.GB_PATH_PER_BEAM
-    W, K = args.warmup, args.steps
-    S = W + 2 * K
+    W = args.warmup
+    K = args.steps if args.steps > 0 else wl.interval
+    S = W + (K if args.no_e2e else 2 * K)
+    C, Hq, Hkv, D, NL = wl.beams, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.num_layers
+    delta = wl.interval
 
     g = GpuRun(wl, device_gen=True, device=str(dev), max_context=wl.context + S + 1, group_min_beams=args.group_min)
     t_build = time.perf_counter()
-    g.build(upto=wl.context)
+    g.build(upto=wl.context - W)            # the schedule's rounds up to here, then plain appends
     torch.cuda.synchronize()
     t_build = time.perf_counter() - t_build
-    C, Hq, Hkv, D, NL = wl.beams, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.num_layers
-    pos0 = g.pos
+    pos0 = g.pos                             # context before the first (warm-up) step
 
-    # Step inputs for every step, generated on the device before timing.
+    def is_round(step: int) -> bool:         # a round follows the step that brings the context to L
+        L = pos0 + step + 1
+        return L > wl.prompt_len and (L - wl.prompt_len) % delta == 0
+
+    round_steps = [i for i in range(S) if is_round(i)]
+    # Step inputs for every step (and hidden states for the round steps), generated before timing.
     qs = torch.empty(S, NL, C, Hq, D, dtype=g.tdt, device=dev)
     ks = torch.empty(S, NL, C, Hkv, D, dtype=g.tdt, device=dev)
     vs = torch.empty_like(ks)
-    hs = torch.empty(S, C, wl.hidden, dtype=g.hidden.dtype, device=dev)
+    hs = torch.empty(max(1, len(round_steps)), C, wl.hidden, dtype=g.hidden.dtype, device=dev)
+    h_index = {s: n for n, s in enumerate(round_steps)}
     for i in range(S):
         for l in range(NL):
             gpu_gen.normal(qs[i, l], wl.kv_dtype, 1, C, Hq * D, [wl.seed, gen.TAG_Q, l, (0, 0, 1), pos0 + i],
@@ -241,31 +270,39 @@ def run_ours(args) -> None:
             for which, dst in ((gen.TAG_KV_K, ks), (gen.TAG_KV_V, vs)):
                 gpu_gen.normal(dst[i, l], wl.kv_dtype, 1, C, Hkv * D, [wl.seed, which, l, (0, 0, 1), pos0 + i],
                                row_scale=g.hscale_dev[l] if g.hscale else None, row_scale_div=D)
-        gpu_gen.normal(hs[i], wl.hidden_dtype, 1, C, wl.hidden, [wl.seed, gen.TAG_HIDDEN, (0, 0, 1), pos0 + i])
+    for s, n in h_index.items():
+        gpu_gen.normal(hs[n], wl.hidden_dtype, 1, C, wl.hidden, [wl.seed, gen.TAG_HIDDEN, (0, 0, 1), pos0 + s + 1])
     out = torch.empty(NL, C, Hq, D, dtype=torch.float32, device=dev)
     pool = g.pool
-
-    def step(i):
-        for l in range(NL):
-            pool.decode_attention(l, qs[i, l], ks[i, l], vs[i, l], wl.attn_scale, out[l], flags)
-        pool.score_probe(hs[i], wl.hidden_dtype, g.w, wl.bias, None, g.scores)
-        pool.prune_branch(wl.K, wl.fanout, wl.warmup, None, g.parent, g.pruned, g.lineage)
-
     stream = torch.cuda.current_stream()
+
+    def step(i, q, k, v, h, prof=None):
+        for l in range(NL):
+            if prof is not None:
+                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_DECODE, *prof["dec"][l])
+                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_GROUPED, *prof["gr"][l])
+            pool.decode_attention(l, q[l], k[l], v[l], wl.attn_scale, out[l], flags)
+        if is_round(i):
+            if prof is not None:
+                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PROBE, *prof["probe"])
+                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PRUNE, *prof["prune"])
+            pool.score_probe(h, wl.hidden_dtype, g.w, wl.bias, None, g.scores)
+            pool.prune_branch(wl.K, wl.fanout, wl.warmup, None, g.parent, g.pruned, g.lineage)
+
     for i in range(W):
-        step(i)
+        step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)])
     torch.cuda.synchronize()
 
-    # Per-kernel events (recorded by the library on this stream around the kernels).
-    def events(n):
-        evs = [torch.cuda.Event(enable_timing=True) for _ in range(n)]
-        for e in evs:
-            e.record(stream)
-        return evs
-    n_dec = K * NL
-    dec_a, dec_b = events(n_dec), events(n_dec)
-    gr_a, gr_b = events(n_dec), events(n_dec)
-    pr_a, pr_b, pb_a, pb_b = events(K), events(K), events(K), events(K)
+    # Per-kernel events, recorded by the library on this stream around the kernels.
+    def ev_pair():
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        b.record(stream)
+        return a, b
+    timed_rounds = [i for i in range(W, W + K) if is_round(i)]
+    profs = {i: {"dec": [ev_pair() for _ in range(NL)], "gr": [ev_pair() for _ in range(NL)]} for i in range(W, W + K)}
+    for i in timed_rounds:
+        profs[i]["probe"], profs[i]["prune"] = ev_pair(), ev_pair()
     torch.cuda.synchronize()
     launches0 = B.gb_pool_launch_count(pool.handle)
     clocks = ClockSampler(gpu_id_for_smi(local))
@@ -275,16 +312,8 @@ def run_ours(args) -> None:
     torch.cuda.synchronize()
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
-    for k in range(K):
-        i = W + k
-        B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PRUNE, pr_a[k], pr_b[k])
-        B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PROBE, pb_a[k], pb_b[k])
-        for l in range(NL):
-            B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_DECODE, dec_a[k * NL + l], dec_b[k * NL + l])
-            B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_GROUPED, gr_a[k * NL + l], gr_b[k * NL + l])
-            pool.decode_attention(l, qs[i, l], ks[i, l], vs[i, l], wl.attn_scale, out[l], flags)
-        pool.score_probe(hs[i], wl.hidden_dtype, g.w, wl.bias, None, g.scores)
-        pool.prune_branch(wl.K, wl.fanout, wl.warmup, None, g.parent, g.pruned, g.lineage)
+    for i in range(W, W + K):
+        step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)], profs[i])
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -292,21 +321,22 @@ def run_ours(args) -> None:
     clk = clocks.stop()
     for which in (B.GB_PROF_DECODE, B.GB_PROF_PROBE, B.GB_PROF_PRUNE, B.GB_PROF_GROUPED):
         B.gb_pool_set_profile_events(pool.handle, which, None, None)
-    stats = B.gb_pool_read_step_stats(pool.handle, max_steps=K)  # one record per timed step (layer 0 opens it)
+    stats = B.gb_pool_read_step_stats(pool.handle, max_steps=K)  # one record per timed step
     launches = B.gb_pool_launch_count(pool.handle) - launches0
     elapsed_ms = t_start.elapsed_time(t_end)
     if world > 1:
         t = torch.tensor([elapsed_ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         elapsed_ms = float(t.item())
-    dec_ms = [a.elapsed_time(b) for a, b in zip(dec_a, dec_b)]
-    prune_us = statistics.mean(a.elapsed_time(b) for a, b in zip(pr_a, pr_b)) * 1e3
-    probe_us = statistics.mean(a.elapsed_time(b) for a, b in zip(pb_a, pb_b)) * 1e3
     status = pool.status()
     if status != 0:
         raise RuntimeError(f"device status {status} after the timed steps: the measurement is invalid")
-
-    gr_ms = [a.elapsed_time(b) for a, b in zip(gr_a, gr_b)]
+    dec_ms = [a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["dec"]]
+    gr_ms = [a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["gr"]]
+    prune_us = statistics.mean(profs[i]["prune"][0].elapsed_time(profs[i]["prune"][1]) for i in timed_rounds) * 1e3 \
+        if timed_rounds else None
+    probe_us = statistics.mean(profs[i]["probe"][0].elapsed_time(profs[i]["probe"][1]) for i in timed_rounds) * 1e3 \
+        if timed_rounds else None
     grouped_on = flags != B.GB_PATH_PER_BEAM and wl.kv_dtype == "bf16" and D == 128
 
     # Algorithmic work per launch, from the library's per-step records:
@@ -338,33 +368,35 @@ def run_ours(args) -> None:
                                 "frac_hbm": gr_bytes / gr_avg_s / 1e9 / peak, "flops": gr_flops,
                                 "tflops": gr_flops / gr_avg_s / 1e12, "frac_tensor": gr_flops / gr_avg_s / 1e12 / tpeak,
                                 "segments": statistics.mean(int(s[4]) for s in stats),
-                                "tiles": statistics.mean(int(s[5]) for s in stats)}
+                                "work_units": statistics.mean(int(s[5]) * Hkv for s in stats)}
     dominant = "k_grouped" if "k_grouped" in kernels and gr_avg_s > dec_avg_s else "k_decode"
     if dominant == "k_decode":
         roofline = {"bound": "hbm", "kernel": "k_decode (split-KV decode)", "achieved": achieved, "peak": peak,
-                    "unit": "GB/s", "frac": achieved / peak, "traffic": None, "bytes_per_launch": dec_bytes,
+                    "unit": "GB/s", "frac": achieved / peak, "traffic": captured_traffic("k_decode", wl.name, args.flags), "bytes_per_launch": dec_bytes,
                     "peak_source": f"{peak_src} hbm_gbs"}
     else:
         kg = kernels["k_grouped"]
         if kg["frac_tensor"] >= kg["frac_hbm"]:
             roofline = {"bound": "tensor", "kernel": "k_grouped (tcgen05 shared-prefix)", "achieved": kg["tflops"],
-                        "peak": tpeak, "unit": "TFLOP/s", "frac": kg["frac_tensor"], "traffic": None,
+                        "peak": tpeak, "unit": "TFLOP/s", "frac": kg["frac_tensor"], "traffic": captured_traffic("k_grouped", wl.name, args.flags),
                         "flops_per_launch": gr_flops, "peak_source": f"{tpeak_src} bf16_tflops"}
         else:
             roofline = {"bound": "hbm", "kernel": "k_grouped (tcgen05 shared-prefix)", "achieved": kg["gbps"],
-                        "peak": peak, "unit": "GB/s", "frac": kg["frac_hbm"], "traffic": None,
+                        "peak": peak, "unit": "GB/s", "frac": kg["frac_hbm"], "traffic": captured_traffic("k_grouped", wl.name, args.flags),
                         "bytes_per_launch": gr_bytes, "peak_source": f"{peak_src} hbm_gbs"}
 
     value = world * C * K / (elapsed_ms / 1e3)
     ms_per_step = elapsed_ms / K
 
-    # End to end through the C ABI with host buffers: inputs copied in from pinned memory and
-    # outputs read back every step, inside the timed region.
+    # End to end through the C ABI with host buffers: each step's inputs copied in from pinned
+    # memory and its outputs read back, inside the timed region.
     e2e = None
     if not args.no_e2e:
         sl = slice(W + K, W + 2 * K)
-        hq, hk, hv, hh = (t[sl].cpu().pin_memory() for t in (qs, ks, vs, hs))
-        q_d, k_d, v_d, h_d = (torch.empty_like(t[0]) for t in (qs, ks, vs, hs))
+        hq, hk, hv = (t[sl].cpu().pin_memory() for t in (qs, ks, vs))
+        hh = hs.cpu().pin_memory()
+        q_d, k_d, v_d = (torch.empty_like(t[0]) for t in (qs, ks, vs))
+        h_d = torch.empty_like(hs[0])
         o_h = torch.empty(out.shape, dtype=out.dtype).pin_memory()
         s_h = torch.empty(C, dtype=torch.float32).pin_memory()
         p_h = torch.empty(C, dtype=torch.int32).pin_memory()
@@ -374,21 +406,23 @@ def run_ours(args) -> None:
         if world > 1:
             dist.barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        h2d = d2h = 0
         e0.record(stream)
-        for k in range(K):
-            q_d.copy_(hq[k], non_blocking=True)
-            k_d.copy_(hk[k], non_blocking=True)
-            v_d.copy_(hv[k], non_blocking=True)
-            h_d.copy_(hh[k], non_blocking=True)
-            for l in range(NL):
-                pool.decode_attention(l, q_d[l], k_d[l], v_d[l], wl.attn_scale, out[l], flags)
-            pool.score_probe(h_d, wl.hidden_dtype, g.w, wl.bias, None, g.scores)
-            pool.prune_branch(wl.K, wl.fanout, wl.warmup, None, g.parent, g.pruned, g.lineage)
+        for n, i in enumerate(range(W + K, W + 2 * K)):
+            q_d.copy_(hq[n], non_blocking=True)
+            k_d.copy_(hk[n], non_blocking=True)
+            v_d.copy_(hv[n], non_blocking=True)
+            h2d += sum(t[n].numel() * t.element_size() for t in (hq, hk, hv))
+            if is_round(i):
+                h_d.copy_(hh[h_index[i]], non_blocking=True)
+                h2d += hh[0].numel() * hh.element_size()
+            step(i, q_d, k_d, v_d, h_d)
             o_h.copy_(out, non_blocking=True)
-            s_h.copy_(g.scores, non_blocking=True)
-            p_h.copy_(g.parent, non_blocking=True)
-            pr_h.copy_(g.pruned, non_blocking=True)
-            ln_h.copy_(g.lineage, non_blocking=True)
+            d2h += o_h.numel() * o_h.element_size()
+            if is_round(i):
+                for host, dev_t in ((s_h, g.scores), (p_h, g.parent), (pr_h, g.pruned), (ln_h, g.lineage)):
+                    host.copy_(dev_t, non_blocking=True)
+                    d2h += host.numel() * host.element_size()
         e1.record(stream)
         torch.cuda.synchronize()
         e_ms = e0.elapsed_time(e1)
@@ -396,11 +430,11 @@ def run_ours(args) -> None:
             t = torch.tensor([e_ms], device=dev)
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             e_ms = float(t.item())
-        h2d = sum(t[0].numel() * t.element_size() for t in (hq, hk, hv, hh))
-        d2h = sum(t.numel() * t.element_size() for t in (o_h, s_h, p_h, pr_h, ln_h))
-        e2e = {"value": world * C * K / (e_ms / 1e3), "unit": "beam-tokens/s", "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h), "ms_per_step": e_ms / K}
-        status = status or pool.status()
+        e2e = {"value": world * C * K / (e_ms / 1e3), "unit": "beam-tokens/s", "h2d_bytes_per_step": int(h2d // K),
+               "d2h_bytes_per_step": int(d2h // K), "ms_per_step": e_ms / K}
+        status = pool.status()
+        if status != 0:
+            raise RuntimeError(f"device status {status} after the e2e steps: the measurement is invalid")
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -411,11 +445,13 @@ def run_ours(args) -> None:
             "value": value, "unit": "beam-tokens/s", "n_gpus": world, "steps": K, "warmup": W,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": wl.kv_dtype, "data": "synthetic (seeded counter-based generator, generated on device)",
-            "config": {"workload": wl.name, "beams": C, "context_at_start": pos0, "context_at_end": pos0 + K,
+            "config": {"workload": wl.name, "beams": C, "context_at_start": pos0 + W, "context_at_end": pos0 + W + K,
                        "layers": NL, "heads": f"{Hq}/{Hkv}", "head_dim": D, "page_size": wl.page_size,
-                       "kv_dtype": wl.kv_dtype, "tournament": f"K={wl.K} fanout={wl.fanout} every step",
+                       "kv_dtype": wl.kv_dtype,
+                       "schedule": f"decode every step; probe + tournament (K={wl.K}, fanout {wl.fanout}) every "
+                                   f"{delta} tokens: {len(timed_rounds)} round(s) in the timed window",
                        "path": args.flags, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                       "l2": f"inputs larger than L2: {C * pos0 * kv_tok / 2**30:.2f} GiB of KV read per step",
+                       "l2": f"inputs larger than L2: {eff_bytes / 2**30:.2f} GiB of per-beam KV reads per step",
                        "tree_build_s": round(t_build, 2)},
             "attention_us": (dec_avg_s + gr_avg_s) * 1e6,
             "attention_tbps": eff_bytes / (dec_avg_s + gr_avg_s) / 1e12,
