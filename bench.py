@@ -55,7 +55,24 @@ def parse_args():
     ap.add_argument("--cpu-beams", type=int, default=16, help="beams per step in the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--beams", type=int, default=0, help="override the workload's beam count (smaller profiling cases)")
+    ap.add_argument("--context", type=int, default=0, help="override the workload's context length")
     return ap.parse_args()
+
+
+def selected_workload(args, rank: int = 0):
+    from workload.configs import BY_INDEX
+    wl = BY_INDEX[args.config - 1]
+    over = {"seed": wl.seed + rank}
+    if args.beams:
+        over["beams"] = args.beams
+        over["K"] = max(1, round(wl.K * args.beams / wl.beams))
+    if args.context:
+        over["context"] = args.context
+    wl = dataclasses.replace(wl, **over)
+    if args.beams or args.context:
+        wl = dataclasses.replace(wl, name=f"{wl.name}[beams={wl.beams},context={wl.context}]")
+    return wl
 
 
 # ---------------------------------------------------------------------------
@@ -237,7 +254,7 @@ def run_ours(args) -> None:
         dist.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    wl = dataclasses.replace(BY_INDEX[args.config - 1], seed=BY_INDEX[args.config - 1].seed + rank)
+    wl = selected_workload(args, rank)
     flags = B.GB_PATH_AUTO if args.flags == "auto" else B.GB_PATH_PER_BEAM
     W = args.warmup
     K = args.steps if args.steps > 0 else wl.interval
@@ -478,9 +495,9 @@ def run_reference(args) -> None:
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    from workload.configs import BY_INDEX
-    wl = BY_INDEX[args.config - 1]
-    W, K = args.warmup, args.steps
+    wl = selected_workload(args)
+    W = args.warmup
+    K = args.steps if args.steps > 0 else wl.interval
     # Each step: a bounded sample (a few beams) so W + K steps end within minutes.
     per_step_beams = max(1, min(args.cpu_beams, 16))
     res = oracle_sample(wl, W + K, per_step_beams)

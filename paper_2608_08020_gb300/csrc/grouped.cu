@@ -5,24 +5,37 @@
 // read once for all of them and Q.K^T and P.V become dense contractions:
 //   S[128 x 64]  = Q[128 x 128] . K_tile^T      (tcgen05.mma kind::f16, fp32 in TMEM)
 //   O[128 x 128] += P[128 x 64] . V_tile         (P in bf16 from the softmax)
-// over 64-token tiles of the segment.  Each unit of work is (segment, KV head,
-// 128-row query tile); a persistent grid of one CTA per SM walks the flat unit list.
-// Results are unnormalised partials (m, l, o) per (beam, depth, head) merged by the
-// combine kernel with the beam's per-beam remainder.
+// over 64-token tiles.  A unit of work is (segment, KV head, 128-row query tile,
+// token split); a persistent grid of one CTA per SM walks the flat unit list, and
+// the tiles of all of a CTA's units form one continuous pipeline.
 //
-// Shared memory (1024-byte aligned, 128-byte swizzle everywhere):
-//   Q   two [128 rows][64 dims] blocks (K-major A operand)             32 KiB
-//   K,V per stage: two [64 tokens][64 dims] blocks each               32 KiB x 2 stages
-//   P   one [128 rows][64 tokens] block (K-major A operand)           16 KiB
-// K/V chunks of 16 tokens arrive by 2D TMA loads (box 64 dims x 16 rows) from a
-// tensor map over the whole pool; chunks past the segment end load out of bounds
-// and are zero-filled.  V is the B operand in MN-major form (dims contiguous).
+// Warp roles (192 threads):
+//   warps 0-3  softmax: thread r owns query row r (TMEM lane r); reads S, keeps the
+//              running max / sum, writes P (bf16) and, at the end of a unit, the
+//              unnormalised partial record (m, l, o) of its row;
+//   warp 4     producer: gathers the next unit's query rows into one of two Q
+//              buffers and streams K/V tiles through a 4-stage ring by 2D TMA;
+//   warp 5     MMA issuer: polls both queues and issues S(n+1) or P.V(n), whichever
+//              is ready first, so the tensor core works while the softmax warps
+//              handle tile n.
+// Handshakes are mbarriers: full/empty per K/V stage, q_full/q_empty per Q buffer,
+// s_full/s_free and p_full/p_empty per double-buffered S (TMEM) and P (smem) tile.
+// MMA completion is signalled with tcgen05.commit.
 //
-// Softmax: thread r owns row r (TMEM lane r).  The running maximum is only raised
-// when a tile's maximum exceeds it by more than 8 (base 2); smaller increases are
-// absorbed in p <= 2^8, so O in TMEM is rescaled rarely.  Every mbarrier wait is
-// bounded; on timeout the CTA records GB_ERR_TIMEOUT, drains its own copies and
-// MMAs (bounded), frees its tensor memory and leaves.
+// Shared memory (dynamic only, 1024-byte aligned, 128-byte swizzle everywhere):
+//   Q   2 x two [128 rows][64 dims] blocks (K-major A operand)        64 KiB
+//   K,V 4 stages x (two [64 tokens][64 dims] blocks each)             128 KiB
+//   P   2 x one [128 rows][64 tokens] block (K-major A operand)       32 KiB
+// K/V arrive as 16-token chunks (TMA box 64 dims x 16 rows) from a tensor map over
+// the whole pool; chunks past the unit's tokens load out of bounds and are zero-
+// filled.  V is the B operand in MN-major form (dims contiguous).
+//
+// Softmax (base 2): the running max is raised only when a tile's max exceeds it by
+// more than 8; smaller increases are absorbed in p <= 2^8, so O is rescaled rarely.
+// Each score costs one FFMA and one ex2.approx; the sum l is kept in fp32.
+// Every wait is bounded; on timeout the CTA records GB_ERR_TIMEOUT, every role stops
+// issuing, waits (bounded) for its own outstanding copies and MMAs, the tensor
+// memory is freed and the CTA leaves.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -34,15 +47,30 @@ namespace {
 constexpr int kRows = 128;     // query rows per tile (MMA M)
 constexpr int kTok = 64;       // tokens per K/V tile (MMA N of Q.K^T, K of P.V)
 constexpr int kStages = 4;
-constexpr int kThreads = 128;
-constexpr uint32_t kTmemCols = 256;  // S: columns [0, 64), O: [128, 256)
+constexpr int kThreads = 192;
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr uint32_t kTmemCols = 256;  // S0: [0, 64), S1: [64, 128), O: [128, 256)
 
-constexpr int kQ = 0;
-constexpr int kKV = 32768;
-constexpr int kStage = 32768;        // K 16 KiB + V 16 KiB
-constexpr int kP = kKV + kStages * kStage;
-constexpr int kSmem = kP + 16384;
-constexpr int kSmemAlloc = kSmem + 1024;
+constexpr int kQ = 0;                // 2 buffers x 32 KiB
+constexpr int kKV = 65536;           // 4 stages x 32 KiB (K 16 KiB + V 16 KiB)
+constexpr int kStage = 32768;
+constexpr int kP = kKV + kStages * kStage;  // 2 buffers x 16 KiB
+constexpr int kBar = kP + 32768;     // mbarriers and control words
+constexpr int kSmem = kBar + 256;
+
+// Control area (8-byte mbarriers, then words).
+constexpr int kBarFull = 0;          // [kStages]
+constexpr int kBarEmpty = kBarFull + 8 * kStages;
+constexpr int kBarQFull = kBarEmpty + 8 * kStages;   // [2]
+constexpr int kBarQEmpty = kBarQFull + 16;           // [2]
+constexpr int kBarSFull = kBarQEmpty + 16;           // [2]
+constexpr int kBarSFree = kBarSFull + 16;            // [2]
+constexpr int kBarPFull = kBarSFree + 16;            // [2]
+constexpr int kBarPEmpty = kBarPFull + 16;           // [2]
+constexpr int kWordTmem = kBarPEmpty + 16;
+constexpr int kWordAbort = kWordTmem + 4;
+static_assert(kWordAbort + 4 <= 256, "control area");
 
 __device__ __forceinline__ uint32_t swz(int r, int col) {  // byte offset of (row, col) in a [rows][64] bf16 SW128 block
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((((col >> 3) ^ (r & 7))) << 4) + (col & 7) * 2);
@@ -72,6 +100,10 @@ __device__ __forceinline__ void mma(uint32_t tmem_d, uint64_t a, uint64_t b, uin
 
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ void tma_2d(uint32_t dst, const CUtensorMap* tm, int x, int y, uint32_t bar) {
@@ -115,235 +147,364 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* f) {
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
+// Everything a role needs to know about one unit of work.
+struct Unit {
+  int h, s, t, sp, tok_base, Ts, ntok, seg_i0, rep, g, moff;
+};
+
+__device__ __forceinline__ Unit load_unit(const PoolView& v, long long u) {
+  Unit x;
+  const int tq = (int)(u / v.Hkv);
+  x.h = (int)(u % v.Hkv);
+  x.s = v.seg_tile_seg[tq];
+  x.t = v.seg_tile_t[tq];
+  x.sp = v.seg_tile_split[tq];
+  const int split = v.ctl[kCtlSegSplit];
+  x.tok_base = x.sp * split;
+  x.Ts = min(v.seg_len[x.s] * v.P - x.tok_base, split);
+  x.ntok = (x.Ts + kTok - 1) / kTok;
+  x.seg_i0 = v.seg_i0[x.s];
+  x.rep = v.seg_rep[x.s];
+  x.g = v.seg_g[x.s];
+  x.moff = v.seg_mem_off[x.s];
+  return x;
+}
+
+// Bounded wait that also gives up when another role aborted.
+__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 63) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        return false;
+      }
+    }
+  }
+}
+
 template <int G>
 __global__ void __launch_bounds__(kThreads, 1)
     k_grouped(PoolView v, const __grid_constant__ CUtensorMap tm, int layer, const __nv_bfloat16* __restrict__ q,
               float qscale, long long total_rows) {
-  extern __shared__ __align__(1024) unsigned char smem_raw[];
-  unsigned char* sm = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  __shared__ __align__(8) uint64_t bar_full[kStages];
-  __shared__ __align__(8) uint64_t bar_s, bar_pv;
-  __shared__ uint32_t tmem_slot;
-  __shared__ int s_abort;
-
+  extern __shared__ __align__(1024) unsigned char sm[];
   if (v.ctl[kCtlStepOk] == 0) return;
-  const int ntiles_q = v.ctl[kCtlSegTiles];
-  const long long units = (long long)ntiles_q * v.Hkv;
+  const long long units = (long long)v.ctl[kCtlSegTiles] * v.Hkv;
   if (blockIdx.x >= units) return;
-
-  const int tid = threadIdx.x, warp = tid >> 5;
-  const uint32_t sbase = smem_addr(sm);
-  const uint32_t bfull0 = smem_addr(&bar_full[0]);
-  const uint32_t bs = smem_addr(&bar_s), bpv = smem_addr(&bar_pv);
-  if (tid == 0) {
-    for (int i = 0; i < kStages; ++i) mbar_init(bfull0 + 8 * i, 1);
-    mbar_init(bs, 1);
-    mbar_init(bpv, 1);
-    fence_mbar_init();
-    s_abort = 0;
+  if (smem_addr(sm) & 1023) {  // the swizzled layouts need a 1024-byte aligned base
+    if (threadIdx.x == 0) set_status(v.ctl, GB_ERR_UNSUPPORTED);
+    return;
   }
-  if (warp == 0) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&tmem_slot)),
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t sbase = smem_addr(sm);
+  const uint32_t ctl = sbase + kBar;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + kBar + kWordAbort);
+  if (tid == 0) {
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(ctl + kBarFull + 8 * i, 1);
+      mbar_init(ctl + kBarEmpty + 8 * i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(ctl + kBarQFull + 8 * i, 1);
+      mbar_init(ctl + kBarQEmpty + 8 * i, 1);
+      mbar_init(ctl + kBarSFull + 8 * i, 1);
+      mbar_init(ctl + kBarSFree + 8 * i, 4);
+      mbar_init(ctl + kBarPFull + 8 * i, 4);
+      mbar_init(ctl + kBarPEmpty + 8 * i, 1);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(ctl + kWordTmem),
                  "r"(kTmemCols));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = tmem_slot;
-  const uint32_t tS = tmem, tO = tmem + 128;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+  const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(sm + kBar + kWordTmem);
+  const long long stride = gridDim.x;
+  constexpr int members_per_tile = kRows / G;
 
-  constexpr uint32_t ID_S = idesc(kTok, false);
-  constexpr uint32_t ID_PV = idesc(128, true);
-  const long long rows_per_kvhead = (long long)v.P;  // tensor-map rows of one (layer, page, kv, head) slab
-
-  // Per-CTA pipeline counters (continue across units).
-  uint32_t loads_issued = 0, loads_used = 0, s_done = 0, pv_done = 0;
-  bool timed_out = false;
-
-  auto issue_tile = [&](int seg_i0, int tok_base, int rep, int h, int Ts, int j, uint32_t stage) {
-    // Tokens [64j, 64j+64) of the segment: four 16-token chunks, K and V, two 64-dim halves.
-    const uint32_t bar = bfull0 + 8 * stage;
-    mbar_arrive_expect_tx(bar, kStage);
-    const uint32_t dst0 = sbase + kKV + stage * kStage;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int tk = tok_base + j * kTok + c * 16;  // token within the segment
-      long long yk = total_rows, yv = total_rows;  // out of bounds: zero fill
-      if (j * kTok + c * 16 < Ts) {
-        int page = v.tables[(size_t)rep * v.max_pages + seg_i0 + tk / v.P];
-        if (page < 0 || page >= v.num_pages) {
-          set_status(v.ctl, GB_ERR_INVALID);
-          page = 0;
-        }
-        const long long slab = (((long long)layer * v.num_pages + page) * 2) * v.Hkv + h;
-        yk = slab * rows_per_kvhead + tk % v.P;
-        yv = (slab + v.Hkv) * rows_per_kvhead + tk % v.P;
-      }
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        tma_2d(dst0 + half * 8192 + c * 2048, &tm, half * 64, (int)yk, bar);
-        tma_2d(dst0 + 16384 + half * 8192 + c * 2048, &tm, half * 64, (int)yv, bar);
-      }
-    }
-  };
-
-  for (long long u = blockIdx.x; u < units && !timed_out; u += gridDim.x) {
-    const int tq = (int)(u / v.Hkv), h = (int)(u % v.Hkv);
-    const int s = v.seg_tile_seg[tq], t = v.seg_tile_t[tq], sp = v.seg_tile_split[tq];
-    const int split = v.ctl[kCtlSegSplit];
-    const int tok_base = sp * split;
-    const int seg_i0 = v.seg_i0[s], rep = v.seg_rep[s], g = v.seg_g[s], moff = v.seg_mem_off[s];
-    const int Ts = min(v.seg_len[s] * v.P - tok_base, split);  // tokens of this split
-    const int ntok = (Ts + kTok - 1) / kTok;
-    constexpr int members_per_tile = kRows / G;
-
-    // Q tile: row r = (member, query head of this KV head), zero rows past the members.
-    {
-      const int r = tid;
-      const int m = t * members_per_tile + r / G, gg = r % G;
-      const bool valid = m < g;
-      const int bk = valid ? v.seg_members[moff + m] : 0;
-      const int b = bk / kMaxSegDepth;
-      const uint4* qrow = reinterpret_cast<const uint4*>(q + ((size_t)b * v.Hq + (size_t)h * G + gg) * 128);
-#pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        const uint4 x = valid ? qrow[c] : make_uint4(0, 0, 0, 0);
-        *reinterpret_cast<uint4*>(sm + kQ + (c >> 3) * 16384 + swz(r, (c & 7) * 8)) = x;
-      }
-    }
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-
-    if (tid == 0) {
-      for (int j = 0; j < kStages && j < ntok; ++j) issue_tile(seg_i0, tok_base, rep, h, Ts, j, (loads_issued + j) % kStages);
-    }
-    uint32_t issued_here = ntok < kStages ? ntok : kStages;
-
-    // S(0)
-    auto issue_s = [&](uint32_t stage) {
-      const uint32_t kb = sbase + kKV + stage * kStage;
-#pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint64_t a = sdesc(sbase + kQ + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-        const uint64_t b = sdesc(kb + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024);
-        mma(tS, a, b, ID_S, kk > 0);
-      }
-      mma_commit(bs);
-    };
-    if (tid == 0) {
-      const uint32_t st = loads_issued % kStages;
-      if (!mbar_wait_bounded(bfull0 + 8 * st, (loads_issued / kStages) & 1, kWaitLimitNs)) {
-        s_abort = 1;
-      } else {
-        tc_fence_after();
-        issue_s(st);
-      }
-    }
-
-    float m_ref = -INFINITY, l = 0.f;
-    for (int j = 0; j < ntok; ++j) {
-      const uint32_t gj = loads_used + j;           // global tile counter of this CTA
-      const uint32_t stage = gj % kStages;
-      // Wait for S(j).
-      if (!mbar_wait_bounded(bs, s_done & 1, kWaitLimitNs)) { timed_out = true; }
-      if (__syncthreads_or(timed_out || s_abort)) { timed_out = true; break; }
-      ++s_done;
-      tc_fence_after();
-      float sv[kTok];
-      tmem_ld32(tS + lane_base + 0, sv);
-      tmem_ld32(tS + lane_base + 32, sv + 32);
-      float mt = -INFINITY;
-#pragma unroll
-      for (int c = 0; c < kTok; ++c) {
-        const bool ok = j * kTok + c < Ts;
-        sv[c] = ok ? sv[c] * qscale : -INFINITY;
-        mt = fmaxf(mt, sv[c]);
-      }
-      // P.V of the previous tile must be done before P and O are touched and its stage refilled.
-      if (j > 0) {
-        if (!mbar_wait_bounded(bpv, pv_done & 1, kWaitLimitNs)) timed_out = true;
-        if (__syncthreads_or(timed_out)) { timed_out = true; break; }
-        ++pv_done;
-        tc_fence_after();
-        if (tid == 0 && j - 1 + kStages < ntok) {
-          issue_tile(seg_i0, tok_base, rep, h, Ts, j - 1 + kStages, (gj - 1) % kStages);
-          ++issued_here;
-        }
-      }
-      const bool raise = mt > m_ref + 8.f;
-      if (j > 0 && __any_sync(0xffffffffu, raise)) {
-        const float alpha = raise ? exp2f(m_ref - mt) : 1.f;
+  if (warp == kProducerWarp) {
+    // ------------------------------------------------------------------ producer
+    if (lane == 0) asm volatile("prefetch.tensormap [%0];" ::"l"(&tm) : "memory");
+    uint32_t n = 0;  // tiles issued
+    int uidx = 0;    // units started
+    for (long long u = blockIdx.x; u < units && !*abort_flag; u += stride, ++uidx) {
+      const Unit x = load_unit(v, u);
+      const int qb = uidx & 1;
+      if (uidx >= 2 && !wait_or_abort(ctl + kBarQEmpty + 8 * qb, ((uidx - 2) >> 1) & 1, abort_flag)) break;
+      // Query rows: row r = (member, query head of this KV head); zero rows past the members.
+      unsigned char* qdst = sm + kQ + qb * 32768;
 #pragma unroll 1
-        for (int c0 = 0; c0 < 128; c0 += 32) {
-          float o[32];
-          tmem_ld32(tO + lane_base + c0, o);
+      for (int r = lane; r < kRows; r += 32) {
+        const int m = x.t * members_per_tile + r / G, gg = r % G;
+        const bool valid = m < x.g;
+        const int b = valid ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
+        const uint4* qrow = reinterpret_cast<const uint4*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
+        uint4 buf[16];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] *= alpha;
-          tmem_st32(tO + lane_base + c0, o);
-        }
-        if (raise) l *= alpha;
-      }
-      if (raise) m_ref = mt;
-      // p = 2^(s - m_ref) in bf16 into the P tile (row = tid), l accumulates the same rounded values.
+        for (int c = 0; c < 16; ++c) buf[c] = valid ? qrow[c] : make_uint4(0, 0, 0, 0);
 #pragma unroll
-      for (int c = 0; c < kTok; c += 8) {
-        __nv_bfloat162 pr[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          pr[i] = __floats2bfloat162_rn(exp2f(sv[c + 2 * i] - m_ref), exp2f(sv[c + 2 * i + 1] - m_ref));
-          const float2 back = __bfloat1622float2(pr[i]);
-          l += back.x + back.y;
-        }
-        *reinterpret_cast<uint4*>(sm + kP + swz(tid, c)) = *reinterpret_cast<const uint4*>(pr);
+        for (int c = 0; c < 16; ++c) *reinterpret_cast<uint4*>(qdst + (c >> 3) * 16384 + swz(r, (c & 7) * 8)) = buf[c];
       }
       fence_proxy_async_smem();
-      tc_fence_before();
-      __syncthreads();
-      if (tid == 0) {
-        tc_fence_after();
-        const uint32_t vb = sbase + kKV + stage * kStage + 16384;
-#pragma unroll
-        for (int kk = 0; kk < kTok / 16; ++kk) {
-          const uint64_t a = sdesc(sbase + kP + kk * 32, 16, 1024);
-          const uint64_t b = sdesc(vb + kk * 2048, 8192, 1024);
-          mma(tO, a, b, ID_PV, (j > 0 || kk > 0) ? 1u : 0u);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ctl + kBarQFull + 8 * qb);
+      // K/V tiles of the unit.  The page ids of the next 32 chunks (16 tokens each) are
+      // loaded by the 32 lanes at once and handed to lane 0 by shuffle.
+      int page_l = 0;
+      for (int j = 0; j < x.ntok; ++j, ++n) {
+        const uint32_t st = n % kStages;
+        const int cb = j * 4;  // first chunk of the tile
+        if ((cb & 31) == 0) {
+          const int tl = (cb + lane) * 16;
+          page_l = tl < x.Ts ? v.tables[(size_t)x.rep * v.max_pages + x.seg_i0 + (x.tok_base + tl) / v.P] : 0;
         }
-        mma_commit(bpv);
-        if (j + 1 < ntok) {
-          const uint32_t st = (gj + 1) % kStages;
-          if (!mbar_wait_bounded(bfull0 + 8 * st, ((gj + 1) / kStages) & 1, kWaitLimitNs)) {
-            s_abort = 1;
-          } else {
-            tc_fence_after();
-            issue_s(st);
+        // Lanes 0..3 compute the tensor-map rows of chunk c = lane (K and V); lane 0 issues.
+        int yk = (int)total_rows, yv = (int)total_rows;  // out of bounds: zero fill
+        {
+          const int c = lane & 3;
+          const int page_c = __shfl_sync(0xffffffffu, page_l, (cb + c) & 31);
+          const int tl = j * kTok + c * 16;  // token within the unit
+          if (tl < x.Ts) {
+            const int tk = x.tok_base + tl;  // token within the segment
+            int page = page_c;
+            if (page < 0 || page >= v.num_pages) {
+              if (lane < 4) set_status(v.ctl, GB_ERR_INVALID);
+              page = 0;
+            }
+            const long long slab = (((long long)layer * v.num_pages + page) * 2) * v.Hkv + x.h;
+            yk = (int)(slab * v.P + tk % v.P);
+            yv = (int)((slab + v.Hkv) * v.P + tk % v.P);
+          }
+        }
+        int ys[8];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          ys[2 * c] = __shfl_sync(0xffffffffu, yk, c);
+          ys[2 * c + 1] = __shfl_sync(0xffffffffu, yv, c);
+        }
+        bool ok = true;
+        if (lane == 0) {
+          if (n >= (uint32_t)kStages) ok = wait_or_abort(ctl + kBarEmpty + 8 * st, ((n / kStages) - 1) & 1, abort_flag);
+          if (ok) {
+            const uint32_t bar = ctl + kBarFull + 8 * st;
+            mbar_arrive_expect_tx(bar, kStage);
+            const uint32_t dst0 = sbase + kKV + st * kStage;
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+              for (int half = 0; half < 2; ++half) {
+                tma_2d(dst0 + half * 8192 + c * 2048, &tm, half * 64, ys[2 * c], bar);
+                tma_2d(dst0 + 16384 + half * 8192 + c * 2048, &tm, half * 64, ys[2 * c + 1], bar);
+              }
+          }
+        }
+        if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) break;
+      }
+    }
+    // Drain: copies still in flight land before the CTA leaves (bounded).
+    if (lane == 0 && *abort_flag) {
+      for (uint32_t k = n > (uint32_t)kStages ? n - kStages : 0; k < n; ++k)
+        mbar_wait_bounded(ctl + kBarFull + 8 * (k % kStages), (k / kStages) & 1, kWaitLimitNs / 8);
+    }
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------------------------ MMA issuer
+    constexpr uint32_t ID_S = idesc(kTok, false);
+    constexpr uint32_t ID_PV = idesc(128, true);
+    uint32_t n_s = 0, n_pv = 0;  // S and P.V tiles issued
+    bool alive = true;
+    // S(n) for the tile at (unit index uidx_s, tile j_s); issued one tile ahead of P.V.
+    long long u_s = blockIdx.x;
+    int uidx_s = 0, j_s = 0;
+    Unit xs{};
+    if (u_s < units) xs = load_unit(v, u_s);
+    // S(n_s) can go when its Q buffer is filled (first tile of a unit), its K/V stage has
+    // landed and the softmax warps are done with S(n_s - 2) in the same TMEM buffer.
+    auto s_ready = [&]() -> bool {
+      const uint32_t st = n_s % kStages, sb = n_s & 1;
+      if (j_s == 0 && !mbar_test(ctl + kBarQFull + 8 * (uidx_s & 1), (uidx_s >> 1) & 1)) return false;
+      if (!mbar_test(ctl + kBarFull + 8 * st, (n_s / kStages) & 1)) return false;
+      return n_s < 2 || mbar_test(ctl + kBarSFree + 8 * sb, ((n_s >> 1) - 1) & 1);
+    };
+    auto issue_s = [&]() {
+      const uint32_t st = n_s % kStages, sb = n_s & 1;
+      tc_fence_after();
+      const uint32_t qa = sbase + kQ + (uidx_s & 1) * 32768;
+      const uint32_t kb = sbase + kKV + st * kStage;
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t a = sdesc(qa + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+        const uint64_t b = sdesc(kb + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024);
+        mma(tmem + sb * 64, a, b, ID_S, kk > 0);
+      }
+      mma_commit(ctl + kBarSFull + 8 * sb);
+      if (j_s + 1 == xs.ntok) mma_commit(ctl + kBarQEmpty + 8 * (uidx_s & 1));  // last read of this Q buffer
+      ++n_s;
+      if (++j_s == xs.ntok) {
+        j_s = 0;
+        ++uidx_s;
+        u_s += stride;
+        if (u_s < units) xs = load_unit(v, u_s);
+      }
+    };
+    if (lane == 0) {
+      // Poll both queues and issue whichever MMA is ready, so P.V(n) never waits behind
+      // the data of tile n+1 and S(n+1) never waits behind the softmax of tile n.
+      long long u_p = blockIdx.x;
+      int j_p = 0;
+      Unit xp = load_unit(v, u_p);
+      uint64_t t_progress = globaltimer_ns();
+      uint32_t spins = 0;
+      while (u_p < units) {
+        bool progressed = false;
+        if (u_s < units && s_ready()) {
+          issue_s();
+          progressed = true;
+        }
+        const uint32_t pb = n_pv & 1, st = n_pv % kStages;
+        if (n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv >> 1) & 1)) {
+          tc_fence_after();
+          const uint32_t pa = sbase + kP + pb * 16384;
+          const uint32_t vb = sbase + kKV + st * kStage + 16384;
+#pragma unroll
+          for (int kk = 0; kk < kTok / 16; ++kk) {
+            const uint64_t a = sdesc(pa + kk * 32, 16, 1024);
+            const uint64_t b = sdesc(vb + kk * 2048, 8192, 1024);
+            mma(tmem + 128, a, b, ID_PV, (j_p > 0 || kk > 0) ? 1u : 0u);
+          }
+          mma_commit(ctl + kBarEmpty + 8 * st);
+          mma_commit(ctl + kBarPEmpty + 8 * pb);
+          ++n_pv;
+          if (++j_p == xp.ntok) {
+            j_p = 0;
+            u_p += stride;
+            if (u_p < units) xp = load_unit(v, u_p);
+          }
+          progressed = true;
+        }
+        if (progressed) {
+          spins = 0;
+        } else if ((++spins & 255) == 0) {
+          const uint64_t now = globaltimer_ns();
+          if (spins == 256) t_progress = now;  // first check after the last progress
+          if (*abort_flag || now - t_progress > kWaitLimitNs) {
+            *abort_flag = 1;
+            alive = false;
+            break;
           }
         }
       }
+      if (!alive) {
+        // Let issued MMAs finish before the tensor memory is freed (bounded).
+        if (n_pv > 0) mbar_wait_bounded(ctl + kBarPEmpty + 8 * ((n_pv - 1) & 1), ((n_pv - 1) >> 1) & 1, kWaitLimitNs / 8);
+        if (n_s > 0) mbar_wait_bounded(ctl + kBarSFull + 8 * ((n_s - 1) & 1), ((n_s - 1) >> 1) & 1, kWaitLimitNs / 8);
+      }
     }
-    if (timed_out) break;
-    // Final P.V, then write this tile's rows.
-    if (!mbar_wait_bounded(bpv, pv_done & 1, kWaitLimitNs)) timed_out = true;
-    if (__syncthreads_or(timed_out)) { timed_out = true; break; }
-    ++pv_done;
-    tc_fence_after();
-    loads_used += ntok;
-    loads_issued += ntok;
-    {
-      const int r = tid;
-      const int m = t * members_per_tile + r / G, gg = r % G;
-      const int bk = m < g ? v.seg_members[moff + m] : 0;
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------------ softmax (warps 0-3)
+    const int r = tid;  // query row / TMEM lane
+    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    uint32_t n = 0;
+    bool alive = true;
+    for (long long u = blockIdx.x; u < units && alive; u += stride) {
+      const Unit x = load_unit(v, u);
+      float m_ref = -INFINITY, l = 0.f;
+      for (int j = 0; j < x.ntok; ++j, ++n) {
+        const uint32_t sb = n & 1;
+        if (!wait_or_abort(ctl + kBarSFull + 8 * sb, (n >> 1) & 1, abort_flag)) { alive = false; break; }
+        tc_fence_after();
+        float sv[kTok];
+        tmem_ld32(tmem + sb * 64 + lane_base, sv);
+        tmem_ld32(tmem + sb * 64 + 32 + lane_base, sv + 32);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(ctl + kBarSFree + 8 * sb);
+        // Only a unit's last tile can reach past its tokens (the same for every thread).
+        if ((j + 1) * kTok > x.Ts) {
+#pragma unroll
+          for (int c = 0; c < kTok; ++c)
+            if (j * kTok + c >= x.Ts) sv[c] = -INFINITY;
+        }
+        // Max on the raw scores; qscale > 0, so it scales to the max in log2 units.
+        float mr0 = sv[0], mr1 = sv[1];
+#pragma unroll
+        for (int c = 2; c < kTok; c += 2) {
+          mr0 = fmaxf(mr0, sv[c]);
+          mr1 = fmaxf(mr1, sv[c + 1]);
+        }
+        const float mt = fmaxf(mr0, mr1) * qscale;
+        const bool raise = mt > m_ref + 8.f;
+        if (j > 0 && __any_sync(0xffffffffu, raise)) {
+          // O must hold P.V(n-1) and nothing newer before it is rescaled.
+          if (!wait_or_abort(ctl + kBarPEmpty + 8 * ((n - 1) & 1), ((n - 1) >> 1) & 1, abort_flag)) {
+            alive = false;
+            break;
+          }
+          tc_fence_after();
+          const float alpha = raise ? exp2f(m_ref - mt) : 1.f;
+#pragma unroll 1
+          for (int c0 = 0; c0 < 128; c0 += 32) {
+            float o[32];
+            tmem_ld32(tmem + 128 + c0 + lane_base, o);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] *= alpha;
+            tmem_st32(tmem + 128 + c0 + lane_base, o);
+          }
+          if (raise) l *= alpha;
+        }
+        if (raise) m_ref = mt;
+        // P in bf16 pairs, computed before the wait for its buffer.
+        const float neg_m = -m_ref;
+        float l0 = 0.f, l1 = 0.f;
+        uint32_t pw[kTok / 2];
+#pragma unroll
+        for (int c = 0; c < kTok; c += 2) {
+          // p = 2^(s * qscale - m); masked scores give 2^-inf = 0.
+          const float p0 = ex2_approx(fmaf(sv[c], qscale, neg_m));
+          const float p1 = ex2_approx(fmaf(sv[c + 1], qscale, neg_m));
+          const __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
+          pw[c / 2] = *reinterpret_cast<const uint32_t*>(&pr);
+          l0 += p0;
+          l1 += p1;
+        }
+        l += l0 + l1;
+        // The P buffer is free once P.V(n-2) has completed.
+        if (n >= 2 && !wait_or_abort(ctl + kBarPEmpty + 8 * sb, ((n >> 1) - 1) & 1, abort_flag)) {
+          alive = false;
+          break;
+        }
+        unsigned char* pdst = sm + kP + sb * 16384;
+#pragma unroll
+        for (int c = 0; c < kTok; c += 8)
+          *reinterpret_cast<uint4*>(pdst + swz(r, c)) = make_uint4(pw[c / 2], pw[c / 2 + 1], pw[c / 2 + 2], pw[c / 2 + 3]);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(ctl + kBarPFull + 8 * sb);
+      }
+      if (!alive) break;
+      // O is final once P.V of the unit's last tile has completed.
+      const uint32_t last = n - 1;
+      if (!wait_or_abort(ctl + kBarPEmpty + 8 * (last & 1), (last >> 1) & 1, abort_flag)) break;
+      tc_fence_after();
+      const int m = x.t * members_per_tile + r / G, gg = r % G;
+      const int bk = m < x.g ? v.seg_members[x.moff + m] : 0;
       const int b = bk / kMaxSegDepth;
-      const int r_idx = v.seg_rec_off[bk] + sp;
-      const bool has = m < g && r_idx < kMaxSegRecords;
-      float* rec = v.grec + (((size_t)b * kMaxSegRecords + r_idx) * v.Hkv + h) * v.record_floats;
+      const int r_idx = v.seg_rec_off[bk] + x.sp;
+      const bool has = m < x.g && r_idx < kMaxSegRecords;
+      float* rec = v.grec + (((size_t)b * kMaxSegRecords + r_idx) * v.Hkv + x.h) * v.record_floats;
 #pragma unroll 1
       for (int c0 = 0; c0 < 128; c0 += 32) {  // warp-collective loads: every lane takes part
         float o[32];
-        tmem_ld32(tO + lane_base + c0, o);
+        tmem_ld32(tmem + 128 + c0 + lane_base, o);
         if (has) {
 #pragma unroll
           for (int i = 0; i < 32; i += 4)
@@ -354,24 +515,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         rec[G * 128 + gg] = m_ref;
         rec[G * 128 + G + gg] = l;
       }
+      tc_fence_before();
     }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
   }
 
-  if (timed_out) {
-    if (tid == 0) {
-      set_status(v.ctl, GB_ERR_TIMEOUT);
-      // Give this CTA's outstanding copies and MMAs a bounded chance to finish before leaving.
-      for (int i = 0; i < kStages; ++i) mbar_wait_bounded(bfull0 + 8 * i, 0, kWaitLimitNs / 8);
-      mbar_wait_bounded(bs, s_done & 1, kWaitLimitNs / 8);
-      mbar_wait_bounded(bpv, pv_done & 1, kWaitLimitNs / 8);
-    }
-  }
+  if (*abort_flag && tid == 0) set_status(v.ctl, GB_ERR_TIMEOUT);
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
+  tc_fence_after();
+  if (warp == kMmaWarp) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
 }
 
 }  // namespace
@@ -408,7 +560,7 @@ template <int G>
 static cudaError_t launch_grouped_t(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(k_grouped<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemAlloc);
+    cudaError_t e = cudaFuncSetAttribute(k_grouped<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
@@ -416,8 +568,8 @@ static cudaError_t launch_grouped_t(gb_pool* pool, int layer, const void* q, flo
   const long long rows = (long long)v.layers * v.num_pages * 2 * v.Hkv * v.P;
   const float qscale = scale * 1.4426950408889634f;
   prof_begin(pool, GB_PROF_GROUPED, s);
-  k_grouped<G><<<pool->num_sms, kThreads, kSmemAlloc, s>>>(
-      v, *reinterpret_cast<const CUtensorMap*>(pool->tmap), layer, static_cast<const __nv_bfloat16*>(q), qscale, rows);
+  k_grouped<G><<<pool->num_sms, kThreads, kSmem, s>>>(v, *reinterpret_cast<const CUtensorMap*>(pool->tmap), layer,
+                                                     static_cast<const __nv_bfloat16*>(q), qscale, rows);
   prof_end(pool, GB_PROF_GROUPED, s);
   pool->launches += 1;
   return cudaGetLastError();
