@@ -50,7 +50,7 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", type=int, default=2, help="workload index 1..5 (default 2: the metric's config)")
     ap.add_argument("--flags", choices=["auto", "per_beam"], default="auto")
-    ap.add_argument("--group-min", type=int, default=0, help="beams a segment needs for the grouped path (0: 16)")
+    ap.add_argument("--group-min", type=int, default=0, help="beams a segment needs for the grouped path (0: library default, 2)")
     ap.add_argument("--cpu-steps", type=int, default=6, help="steps of the oracle sample for cpu_baseline")
     ap.add_argument("--cpu-beams", type=int, default=16, help="beams per step in the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")

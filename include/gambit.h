@@ -72,7 +72,7 @@ typedef struct {
   int64_t num_pages;       /* pages in the pool */
   int max_beams;           /* slots = capacity C of the tournament, <= 1024 */
   int max_pages_per_beam;  /* block-table width */
-  int group_min_beams;     /* grouped path only for segments shared by >= this many beams (0: default 16) */
+  int group_min_beams;     /* grouped path only for segments shared by >= this many beams (0: default 2) */
 } gb_pool_config;
 
 /* Host-side copies of the pool state, for tests and debugging (any member may be NULL). */

@@ -11,24 +11,26 @@
 //
 // Warp roles (192 threads):
 //   warps 0-3  softmax: thread r owns query row r (TMEM lane r); reads S, keeps the
-//              running max / sum, writes P (bf16) and, at the end of a unit, the
-//              unnormalised partial record (m, l, o) of its row;
+//              running max / sum, writes P (bf16) back into the first half of the
+//              tile's S columns and, at the end of a unit, the unnormalised partial
+//              record (m, l, o) of its row;
 //   warp 4     producer: gathers the next unit's query rows into one of two Q
-//              buffers and streams K/V tiles through a 4-stage ring by 2D TMA;
+//              buffers and streams K/V tiles through a 5-stage ring, one 4D TMA per
+//              page for K and one for V;
 //   warp 5     MMA issuer: polls both queues and issues S(n+1) or P.V(n), whichever
-//              is ready first, so the tensor core works while the softmax warps
-//              handle tile n.
+//              is ready first; P.V takes P straight from tensor memory.
 // Handshakes are mbarriers: full/empty per K/V stage, q_full/q_empty per Q buffer,
-// s_full/s_free and p_full/p_empty per double-buffered S (TMEM) and P (smem) tile.
-// MMA completion is signalled with tcgen05.commit.
+// s_full, p_full and pv_done per double-buffered S/P tile.  An S/P buffer is reused by
+// S(n+2) only after P.V(n) has been issued: the tensor core runs a CTA's MMAs in issue
+// order, so P(n) has been read before S(n+2) overwrites it.  MMA completion is signalled
+// with tcgen05.commit.
 //
 // Shared memory (dynamic only, 1024-byte aligned, 128-byte swizzle everywhere):
-//   Q   2 x two [128 rows][64 dims] blocks (K-major A operand)        64 KiB
-//   K,V 4 stages x (two [64 tokens][64 dims] blocks each)             128 KiB
-//   P   2 x one [128 rows][64 tokens] block (K-major A operand)       32 KiB
-// K/V arrive as 16-token chunks (TMA box 64 dims x 16 rows) from a tensor map over
-// the whole pool; chunks past the unit's tokens load out of bounds and are zero-
-// filled.  V is the B operand in MN-major form (dims contiguous).
+//   Q   2 x two [128 rows][64 dims] blocks (K-major A operand)           64 KiB
+//   K,V 5 stages x (K and V: 8-row groups [group][half of D][8][64])     160 KiB
+// Tensor memory: S/P 0 and S/P 1 (64 columns each), O (128 columns).
+// Pages past the unit's tokens load out of bounds and are zero-filled.  V is the B
+// operand in MN-major form (dims contiguous).
 //
 // Softmax (base 2): the running max is raised only when a tile's max exceeds it by
 // more than 8; smaller increases are absorbed in p <= 2^8, so O is rescaled rarely.
@@ -46,17 +48,16 @@ namespace {
 
 constexpr int kRows = 128;     // query rows per tile (MMA M)
 constexpr int kTok = 64;       // tokens per K/V tile (MMA N of Q.K^T, K of P.V)
-constexpr int kStages = 4;
+constexpr int kStages = 5;
 constexpr int kThreads = 192;
 constexpr int kProducerWarp = 4;
 constexpr int kMmaWarp = 5;
-constexpr uint32_t kTmemCols = 256;  // S0: [0, 64), S1: [64, 128), O: [128, 256)
+constexpr uint32_t kTmemCols = 256;  // S/P 0: [0, 64), S/P 1: [64, 128), O: [128, 256)
 
 constexpr int kQ = 0;                // 2 buffers x 32 KiB
-constexpr int kKV = 65536;           // 4 stages x 32 KiB (K 16 KiB + V 16 KiB)
+constexpr int kKV = 65536;           // kStages x 32 KiB (K 16 KiB + V 16 KiB)
 constexpr int kStage = 32768;
-constexpr int kP = kKV + kStages * kStage;  // 2 buffers x 16 KiB
-constexpr int kBar = kP + 32768;     // mbarriers and control words
+constexpr int kBar = kKV + kStages * kStage;  // mbarriers and control words
 constexpr int kSmem = kBar + 256;
 
 // Control area (8-byte mbarriers, then words).
@@ -65,12 +66,12 @@ constexpr int kBarEmpty = kBarFull + 8 * kStages;
 constexpr int kBarQFull = kBarEmpty + 8 * kStages;   // [2]
 constexpr int kBarQEmpty = kBarQFull + 16;           // [2]
 constexpr int kBarSFull = kBarQEmpty + 16;           // [2]
-constexpr int kBarSFree = kBarSFull + 16;            // [2]
-constexpr int kBarPFull = kBarSFree + 16;            // [2]
-constexpr int kBarPEmpty = kBarPFull + 16;           // [2]
-constexpr int kWordTmem = kBarPEmpty + 16;
+constexpr int kBarPFull = kBarSFull + 16;            // [2]
+constexpr int kBarPvDone = kBarPFull + 16;           // [2]
+constexpr int kWordTmem = kBarPvDone + 16;
 constexpr int kWordAbort = kWordTmem + 4;
 static_assert(kWordAbort + 4 <= 256, "control area");
+static_assert(kSmem <= 232448, "shared memory per block");
 
 __device__ __forceinline__ uint32_t swz(int r, int col) {  // byte offset of (row, col) in a [rows][64] bf16 SW128 block
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((((col >> 3) ^ (r & 7))) << 4) + (col & 7) * 2);
@@ -106,10 +107,20 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
-__device__ __forceinline__ void tma_2d(uint32_t dst, const CUtensorMap* tm, int x, int y, uint32_t bar) {
+// P (bf16, in tensor memory) as the A operand.
+__device__ __forceinline__ void mma_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t b, uint32_t id, uint32_t acc) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-      "l"(tm), "r"(x), "r"(y), "r"(bar)
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "r"(tmem_a), "l"(b), "r"(id), "r"(acc));
+}
+
+// One page of one head (K or V) by 4D TMA: coordinates {0, 0, 0, w}, w = first row / 8.
+__device__ __forceinline__ void tma_4d(uint32_t dst, const CUtensorMap* tm, int w, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(
+          dst),
+      "l"(tm), "r"(0), "r"(0), "r"(0), "r"(w), "r"(bar)
       : "memory");
 }
 
@@ -140,6 +151,18 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const float* f) {
       "r"(__float_as_uint(f[20])), "r"(__float_as_uint(f[21])), "r"(__float_as_uint(f[22])), "r"(__float_as_uint(f[23])),
       "r"(__float_as_uint(f[24])), "r"(__float_as_uint(f[25])), "r"(__float_as_uint(f[26])), "r"(__float_as_uint(f[27])),
       "r"(__float_as_uint(f[28])), "r"(__float_as_uint(f[29])), "r"(__float_as_uint(f[30])), "r"(__float_as_uint(f[31]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_st32u(uint32_t taddr, const uint32_t* u) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(u[0]), "r"(u[1]), "r"(u[2]), "r"(u[3]), "r"(u[4]), "r"(u[5]), "r"(u[6]), "r"(u[7]), "r"(u[8]), "r"(u[9]),
+      "r"(u[10]), "r"(u[11]), "r"(u[12]), "r"(u[13]), "r"(u[14]), "r"(u[15]), "r"(u[16]), "r"(u[17]), "r"(u[18]),
+      "r"(u[19]), "r"(u[20]), "r"(u[21]), "r"(u[22]), "r"(u[23]), "r"(u[24]), "r"(u[25]), "r"(u[26]), "r"(u[27]),
+      "r"(u[28]), "r"(u[29]), "r"(u[30]), "r"(u[31])
       : "memory");
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
@@ -211,9 +234,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(ctl + kBarQFull + 8 * i, 1);
       mbar_init(ctl + kBarQEmpty + 8 * i, 1);
       mbar_init(ctl + kBarSFull + 8 * i, 1);
-      mbar_init(ctl + kBarSFree + 8 * i, 4);
       mbar_init(ctl + kBarPFull + 8 * i, 4);
-      mbar_init(ctl + kBarPEmpty + 8 * i, 1);
+      mbar_init(ctl + kBarPvDone + 8 * i, 1);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -233,6 +255,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------------ producer
     if (lane == 0) asm volatile("prefetch.tensormap [%0];" ::"l"(&tm) : "memory");
+    const int ppt = kTok / v.P;                  // pages per K/V tile (1 to 8)
+    const uint32_t page_bytes = (uint32_t)v.P * 256;  // one page of one head: P rows of 256 bytes
+    const int w_oob = (int)(total_rows / 8);     // first row group past the pool: loads zeros
     uint32_t n = 0;  // tiles issued
     int uidx = 0;    // units started
     for (long long u = blockIdx.x; u < units && !*abort_flag; u += stride, ++uidx) {
@@ -256,39 +281,38 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(ctl + kBarQFull + 8 * qb);
-      // K/V tiles of the unit.  The page ids of the next 32 chunks (16 tokens each) are
-      // loaded by the 32 lanes at once and handed to lane 0 by shuffle.
+      // K/V tiles of the unit, one 4D TMA per page for K and one for V.  The page ids of
+      // the next 32 pages are loaded by the 32 lanes at once and handed out by shuffle.
       int page_l = 0;
       for (int j = 0; j < x.ntok; ++j, ++n) {
         const uint32_t st = n % kStages;
-        const int cb = j * 4;  // first chunk of the tile
-        if ((cb & 31) == 0) {
-          const int tl = (cb + lane) * 16;
+        const int pb = j * ppt;  // first page of the tile within the unit
+        if ((pb & 31) == 0) {
+          const int tl = (pb + lane) * v.P;
           page_l = tl < x.Ts ? v.tables[(size_t)x.rep * v.max_pages + x.seg_i0 + (x.tok_base + tl) / v.P] : 0;
         }
-        // Lanes 0..3 compute the tensor-map rows of chunk c = lane (K and V); lane 0 issues.
-        int yk = (int)total_rows, yv = (int)total_rows;  // out of bounds: zero fill
+        // Lane c < ppt computes the row groups of page c (K and V) of this tile.
+        int wk = w_oob, wv = w_oob;
         {
-          const int c = lane & 3;
-          const int page_c = __shfl_sync(0xffffffffu, page_l, (cb + c) & 31);
-          const int tl = j * kTok + c * 16;  // token within the unit
-          if (tl < x.Ts) {
-            const int tk = x.tok_base + tl;  // token within the segment
+          const int c = lane & 7;
+          const int page_c = __shfl_sync(0xffffffffu, page_l, (pb + c) & 31);
+          const int tl = j * kTok + c * v.P;  // token within the unit
+          if (lane < ppt && tl < x.Ts) {
             int page = page_c;
             if (page < 0 || page >= v.num_pages) {
-              if (lane < 4) set_status(v.ctl, GB_ERR_INVALID);
+              set_status(v.ctl, GB_ERR_INVALID);
               page = 0;
             }
             const long long slab = (((long long)layer * v.num_pages + page) * 2) * v.Hkv + x.h;
-            yk = (int)(slab * v.P + tk % v.P);
-            yv = (int)((slab + v.Hkv) * v.P + tk % v.P);
+            wk = (int)(slab * v.P / 8);
+            wv = (int)((slab + v.Hkv) * v.P / 8);
           }
         }
-        int ys[8];
+        int ws[16];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          ys[2 * c] = __shfl_sync(0xffffffffu, yk, c);
-          ys[2 * c + 1] = __shfl_sync(0xffffffffu, yv, c);
+        for (int c = 0; c < 8; ++c) {
+          ws[2 * c] = __shfl_sync(0xffffffffu, wk, c);
+          ws[2 * c + 1] = __shfl_sync(0xffffffffu, wv, c);
         }
         bool ok = true;
         if (lane == 0) {
@@ -298,11 +322,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive_expect_tx(bar, kStage);
             const uint32_t dst0 = sbase + kKV + st * kStage;
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
-#pragma unroll
-              for (int half = 0; half < 2; ++half) {
-                tma_2d(dst0 + half * 8192 + c * 2048, &tm, half * 64, ys[2 * c], bar);
-                tma_2d(dst0 + 16384 + half * 8192 + c * 2048, &tm, half * 64, ys[2 * c + 1], bar);
+            for (int c = 0; c < 8; ++c)
+              if (c < ppt) {
+                tma_4d(dst0 + c * page_bytes, &tm, ws[2 * c], bar);
+                tma_4d(dst0 + 16384 + c * page_bytes, &tm, ws[2 * c + 1], bar);
               }
           }
         }
@@ -320,18 +343,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t ID_PV = idesc(128, true);
     uint32_t n_s = 0, n_pv = 0;  // S and P.V tiles issued
     bool alive = true;
-    // S(n) for the tile at (unit index uidx_s, tile j_s); issued one tile ahead of P.V.
-    long long u_s = blockIdx.x;
+    long long u_s = blockIdx.x;  // the tile of the next S: unit, unit index, tile in unit
     int uidx_s = 0, j_s = 0;
     Unit xs{};
     if (u_s < units) xs = load_unit(v, u_s);
     // S(n_s) can go when its Q buffer is filled (first tile of a unit), its K/V stage has
-    // landed and the softmax warps are done with S(n_s - 2) in the same TMEM buffer.
+    // landed and P.V(n_s - 2), the last reader of its S/P columns, has been issued (the
+    // tensor core executes one CTA's MMAs in issue order).
     auto s_ready = [&]() -> bool {
-      const uint32_t st = n_s % kStages, sb = n_s & 1;
       if (j_s == 0 && !mbar_test(ctl + kBarQFull + 8 * (uidx_s & 1), (uidx_s >> 1) & 1)) return false;
-      if (!mbar_test(ctl + kBarFull + 8 * st, (n_s / kStages) & 1)) return false;
-      return n_s < 2 || mbar_test(ctl + kBarSFree + 8 * sb, ((n_s >> 1) - 1) & 1);
+      if (!mbar_test(ctl + kBarFull + 8 * (n_s % kStages), (n_s / kStages) & 1)) return false;
+      return n_pv + 1 >= n_s;
     };
     auto issue_s = [&]() {
       const uint32_t st = n_s % kStages, sb = n_s & 1;
@@ -341,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
         const uint64_t a = sdesc(qa + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-        const uint64_t b = sdesc(kb + (kk >> 2) * 8192 + (kk & 3) * 32, 16, 1024);
+        const uint64_t b = sdesc(kb + (kk >> 2) * 1024 + (kk & 3) * 32, 16, 2048);
         mma(tmem + sb * 64, a, b, ID_S, kk > 0);
       }
       mma_commit(ctl + kBarSFull + 8 * sb);
@@ -371,16 +393,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t pb = n_pv & 1, st = n_pv % kStages;
         if (n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv >> 1) & 1)) {
           tc_fence_after();
-          const uint32_t pa = sbase + kP + pb * 16384;
           const uint32_t vb = sbase + kKV + st * kStage + 16384;
 #pragma unroll
           for (int kk = 0; kk < kTok / 16; ++kk) {
-            const uint64_t a = sdesc(pa + kk * 32, 16, 1024);
-            const uint64_t b = sdesc(vb + kk * 2048, 8192, 1024);
-            mma(tmem + 128, a, b, ID_PV, (j_p > 0 || kk > 0) ? 1u : 0u);
+            // A = P (bf16 pairs in the S columns, 8 columns per 16 tokens), B = V (MN-major).
+            const uint64_t b = sdesc(vb + kk * 4096, 1024, 2048);
+            mma_ts(tmem + 128, tmem + pb * 64 + kk * 8, b, ID_PV, (j_p > 0 || kk > 0) ? 1u : 0u);
           }
           mma_commit(ctl + kBarEmpty + 8 * st);
-          mma_commit(ctl + kBarPEmpty + 8 * pb);
+          mma_commit(ctl + kBarPvDone + 8 * pb);
           ++n_pv;
           if (++j_p == xp.ntok) {
             j_p = 0;
@@ -403,7 +424,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!alive) {
         // Let issued MMAs finish before the tensor memory is freed (bounded).
-        if (n_pv > 0) mbar_wait_bounded(ctl + kBarPEmpty + 8 * ((n_pv - 1) & 1), ((n_pv - 1) >> 1) & 1, kWaitLimitNs / 8);
+        if (n_pv > 0) mbar_wait_bounded(ctl + kBarPvDone + 8 * ((n_pv - 1) & 1), ((n_pv - 1) >> 1) & 1, kWaitLimitNs / 8);
         if (n_s > 0) mbar_wait_bounded(ctl + kBarSFull + 8 * ((n_s - 1) & 1), ((n_s - 1) >> 1) & 1, kWaitLimitNs / 8);
       }
     }
@@ -419,14 +440,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       float m_ref = -INFINITY, l = 0.f;
       for (int j = 0; j < x.ntok; ++j, ++n) {
         const uint32_t sb = n & 1;
+        const uint32_t sp_addr = tmem + sb * 64 + lane_base;
         if (!wait_or_abort(ctl + kBarSFull + 8 * sb, (n >> 1) & 1, abort_flag)) { alive = false; break; }
         tc_fence_after();
         float sv[kTok];
-        tmem_ld32(tmem + sb * 64 + lane_base, sv);
-        tmem_ld32(tmem + sb * 64 + 32 + lane_base, sv + 32);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(ctl + kBarSFree + 8 * sb);
+        tmem_ld32(sp_addr, sv);
+        tmem_ld32(sp_addr + 32, sv + 32);
         // Only a unit's last tile can reach past its tokens (the same for every thread).
         if ((j + 1) * kTok > x.Ts) {
 #pragma unroll
@@ -444,7 +463,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool raise = mt > m_ref + 8.f;
         if (j > 0 && __any_sync(0xffffffffu, raise)) {
           // O must hold P.V(n-1) and nothing newer before it is rescaled.
-          if (!wait_or_abort(ctl + kBarPEmpty + 8 * ((n - 1) & 1), ((n - 1) >> 1) & 1, abort_flag)) {
+          if (!wait_or_abort(ctl + kBarPvDone + 8 * ((n - 1) & 1), ((n - 1) >> 1) & 1, abort_flag)) {
             alive = false;
             break;
           }
@@ -461,7 +480,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (raise) l *= alpha;
         }
         if (raise) m_ref = mt;
-        // P in bf16 pairs, computed before the wait for its buffer.
+        // P in bf16 pairs over the first 32 columns of this tile's S.
         const float neg_m = -m_ref;
         float l0 = 0.f, l1 = 0.f;
         uint32_t pw[kTok / 2];
@@ -476,16 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           l1 += p1;
         }
         l += l0 + l1;
-        // The P buffer is free once P.V(n-2) has completed.
-        if (n >= 2 && !wait_or_abort(ctl + kBarPEmpty + 8 * sb, ((n >> 1) - 1) & 1, abort_flag)) {
-          alive = false;
-          break;
-        }
-        unsigned char* pdst = sm + kP + sb * 16384;
-#pragma unroll
-        for (int c = 0; c < kTok; c += 8)
-          *reinterpret_cast<uint4*>(pdst + swz(r, c)) = make_uint4(pw[c / 2], pw[c / 2 + 1], pw[c / 2 + 2], pw[c / 2 + 3]);
-        fence_proxy_async_smem();
+        tmem_st32u(sp_addr, pw);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(ctl + kBarPFull + 8 * sb);
@@ -493,7 +503,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!alive) break;
       // O is final once P.V of the unit's last tile has completed.
       const uint32_t last = n - 1;
-      if (!wait_or_abort(ctl + kBarPEmpty + 8 * (last & 1), (last >> 1) & 1, abort_flag)) break;
+      if (!wait_or_abort(ctl + kBarPvDone + 8 * (last & 1), (last >> 1) & 1, abort_flag)) break;
       tc_fence_after();
       const int m = x.t * members_per_tile + r / G, gg = r % G;
       const int bk = m < x.g ? v.seg_members[x.moff + m] : 0;
@@ -528,7 +538,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-// 2D tensor map over the whole pool: rows of D = 128 bf16 (256 bytes), box 64 x 16, 128-byte swizzle.
+// 4D tensor map over the whole pool, which is viewed as rows of D = 128 bf16 (256 bytes):
+// dims {64 dims, 8 rows, 2 halves of D, row groups of 8}, strides {256, 128, 2048} bytes,
+// box {64, 8, 2, P / 8} = one page of one head.  The box lands in shared memory as
+// [row group][half][8 rows][64 dims] with the 128-byte swizzle, so in a 64-token tile the
+// 8-row groups of one half of D sit 2048 bytes apart: the K-major B operand of Q.K^T
+// (SBO 2048, half h at +1024 h) and the MN-major B operand of P.V (LBO 1024, SBO 2048).
 bool make_kv_tensor_map(gb_pool* pool) {
   typedef CUresult (*EncodeFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -542,14 +557,15 @@ bool make_kv_tensor_map(gb_pool* pool) {
       return false;
   }
   const PoolView& v = pool->view;
+  if (v.P % 8 != 0 || kTok % v.P != 0) return false;
   const unsigned long long rows = (unsigned long long)v.layers * v.num_pages * 2 * v.Hkv * v.P;
   if (rows >= (1ull << 31)) return false;
-  cuuint64_t dims[2] = {128, rows};
-  cuuint64_t strides[1] = {256};
-  cuuint32_t box[2] = {64, 16};
-  cuuint32_t es[2] = {1, 1};
+  cuuint64_t dims[4] = {64, 8, 2, rows / 8};
+  cuuint64_t strides[3] = {256, 128, 2048};
+  cuuint32_t box[4] = {64, 8, 2, (cuuint32_t)(v.P / 8)};
+  cuuint32_t es[4] = {1, 1, 1, 1};
   CUtensorMap* m = reinterpret_cast<CUtensorMap*>(pool->tmap);
-  const CUresult r = encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, v.kv, dims, strides, box, es,
+  const CUresult r = encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, v.kv, dims, strides, box, es,
                             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   pool->have_tmap = r == CUDA_SUCCESS;

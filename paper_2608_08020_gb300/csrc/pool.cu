@@ -458,7 +458,7 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   p->next_layer = 0;
   p->step_tokens = 0;
   p->seeded = false;
-  p->group_min = cfg->group_min_beams > 0 ? cfg->group_min_beams : 16;
+  p->group_min = cfg->group_min_beams > 0 ? cfg->group_min_beams : 2;
   PoolView& v = p->view;
   v.layers = cfg->num_layers;
   v.Hq = cfg->num_q_heads;
@@ -514,8 +514,12 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   v.num_sms = p->num_sms;
   v.stats = reinterpret_cast<int*>(m + L.stats);
   v.group_min = p->group_min;
-  // The grouped tensor-core path needs bf16 K/V with D = 128 (kind::f16 MMAs, 128-byte rows).
-  v.grouped = (cfg->kv_dtype == GB_BF16 && cfg->head_dim == 128) ? 1 : 0;
+  // The grouped tensor-core path needs bf16 K/V with D = 128 (kind::f16 MMAs, 128-byte rows)
+  // and pages of 8 to 64 tokens that tile a 64-token K/V tile exactly.
+  v.grouped = (cfg->kv_dtype == GB_BF16 && cfg->head_dim == 128 && cfg->page_size % 8 == 0 &&
+               64 % cfg->page_size == 0)
+                  ? 1
+                  : 0;
   if (v.grouped && !make_kv_tensor_map(p)) v.grouped = 0;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (cudaMemsetAsync(m, 0, L.partials, s) != cudaSuccess ||

@@ -167,15 +167,25 @@ __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
     carry += total;
   }
   __syncthreads();
+  // The list holds at most 9 * max_beams + 2 * SMs entries (each beam sits in at most
+  // kMaxSegDepth segments of >= 2 sharers) and a beam at most kMaxSegDepth + 32 records,
+  // so neither limit is reached for pools of 8 beams or more.  Should the list still
+  // overflow, the step is left entirely to the per-beam path.
+  const bool overflow = carry > cap;
   for (int b = threadIdx.x; b < v.max_beams; b += blockDim.x) {
     int off = 0;
     for (int k = 0; k < v.seg_nseg[b]; ++k) {
       v.seg_rec_off[b * kMaxSegDepth + k] = off;
       off += v.seg_splits[v.seg_bid[b * kMaxSegDepth + k]];
     }
-    v.seg_nrec[b] = off < kMaxSegRecords ? off : kMaxSegRecords;
+    if (overflow || off > kMaxSegRecords) {
+      v.seg_cover[b] = 0;
+      v.seg_nseg[b] = 0;
+      off = 0;
+    }
+    v.seg_nrec[b] = off;
   }
-  if (threadIdx.x == 0) v.ctl[kCtlSegTiles] = carry < cap ? carry : cap;
+  if (threadIdx.x == 0) v.ctl[kCtlSegTiles] = overflow ? 0 : carry;
 }
 
 cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s) {

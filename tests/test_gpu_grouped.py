@@ -18,7 +18,7 @@ pytestmark = pytest.mark.gpu
 
 @pytest.mark.parametrize("beams,group_min,prompt,context,interval,K", [
     (32, 4, 100, 520, 100, 16),     # 32 beams x 4 heads = one 128-row tile for the prompt
-    (64, 16, 200, 700, 150, 32),    # 256 rows = two tiles; group_min as in the default
+    (64, 16, 200, 700, 150, 32),    # 256 rows = two tiles; only the widest segments grouped
     (48, 2, 37, 400, 70, 24),       # small segments, unaligned prompt and forks
 ])
 def test_grouped_matches_oracle(cuda, beams, group_min, prompt, context, interval, K):
