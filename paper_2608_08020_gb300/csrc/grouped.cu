@@ -3,41 +3,44 @@
 // For a segment of pages shared by g beams, the g x G query rows of one KV head
 // (G = Hq / Hkv) are stacked into one 128-row tile, so the segment's K and V are
 // read once for all of them and Q.K^T and P.V become dense contractions:
-//   S[128 x 64]  = Q[128 x 128] . K_tile^T      (tcgen05.mma kind::f16, fp32 in TMEM)
-//   O[128 x 128] += P[128 x 64] . V_tile         (P in bf16 from the softmax)
-// over 64-token tiles.  A unit of work is (segment, KV head, 128-row query tile,
-// token split); a persistent grid of one CTA per SM walks the flat unit list, and
-// the tiles of all of a CTA's units form one continuous pipeline.
+//   S[128 x 128]  = Q[128 x 128] . K_tile^T          (tcgen05.mma kind::f16, fp32 in TMEM)
+//   O_k[128 x 128] += P_k[128 x 64] . V_tile,k        (k = 0, 1: the two 64-token halves)
+// over 128-token tiles.  A unit of work is (segment, KV head, 128-row query tile, token
+// split); a persistent grid of one CTA per SM walks the flat unit list, and the tiles of
+// all of a CTA's units form one continuous pipeline.
 //
-// Warp roles (192 threads):
-//   warps 0-3  softmax: thread r owns query row r (TMEM lane r); reads S, keeps the
-//              running max / sum, writes P (bf16) back into the first half of the
-//              tile's S columns and, at the end of a unit, the unnormalised partial
-//              record (m, l, o) of its row;
-//   warp 4     producer: gathers the next unit's query rows into one of two Q
-//              buffers and streams K/V tiles through a 5-stage ring, one 4D TMA per
-//              page for K and one for V;
-//   warp 5     MMA issuer: polls both queues and issues S(n+1) or P.V(n), whichever
-//              is ready first; P.V takes P straight from tensor memory.
-// Handshakes are mbarriers: full/empty per K/V stage, q_full/q_empty per Q buffer,
-// s_full, p_full and pv_done per double-buffered S/P tile.  An S/P buffer is reused by
-// S(n+2) only after P.V(n) has been issued: the tensor core runs a CTA's MMAs in issue
-// order, so P(n) has been read before S(n+2) overwrites it.  MMA completion is signalled
-// with tcgen05.commit.
+// Warp roles (320 threads):
+//   warps 0-3  softmax group 0 and warps 4-7 softmax group 1: thread r of group k owns
+//              query row r (TMEM lane r) and tokens [64k, 64k + 64) of every tile, with
+//              its own running max m_k, sum l_k and accumulator O_k; it writes P_k (bf16)
+//              over the first 32 of its S columns.  At the end of a unit the two groups
+//              exchange (m, l) through shared memory and each writes half of the merged
+//              unnormalised record (m, l, o) of its row;
+//   warp 8     producer: gathers each unit's query rows into the Q buffer and streams
+//              K/V tiles through a 3-stage ring, one 5D TMA per page (K and V of one
+//              head), issued by several lanes at once;
+//   warp 9     MMA issuer: polls and issues S(n+1) or P.V(n), whichever is ready first;
+//              P.V takes P straight from tensor memory.
+// Handshakes are mbarriers: full/empty per stage, q_full/q_empty, s_full, p_full and
+// pv_done per double-buffered S/P tile, xch_full and o_free per unit.  An S/P buffer is
+// reused by S(n+2) only after P.V(n) has been issued: the tensor core runs a CTA's MMAs
+// in issue order, so P(n) has been read before S(n+2) overwrites it.
 //
 // Shared memory (dynamic only, 1024-byte aligned, 128-byte swizzle everywhere):
-//   Q   2 x two [128 rows][64 dims] blocks (K-major A operand)           64 KiB
-//   K,V 5 stages x (K and V: 8-row groups [group][half of D][8][64])     160 KiB
-// Tensor memory: S/P 0 and S/P 1 (64 columns each), O (128 columns).
-// Pages past the unit's tokens load out of bounds and are zero-filled.  V is the B
-// operand in MN-major form (dims contiguous).
+//   Q     two [128 rows][64 dims] blocks (K-major A operand)                32 KiB
+//   K,V   3 stages x 16 row groups of 8 tokens: [group][K|V][half of D][8][64] 192 KiB
+//   xch   (m, l) of both softmax groups for the unit-end merge                2 KiB
+// In a stage, K's 8-token groups sit 4096 bytes apart (Q.K^T: K-major B, SBO 4096, half
+// of D at +1024) and so do V's (P.V: MN-major B at +2048, LBO 1024, SBO 4096).
+// Tensor memory: S/P 0 and S/P 1 (128 columns each), O_0 and O_1 (128 columns each).
+// Pages past the unit's tokens load out of bounds and are zero-filled.
 //
-// Softmax (base 2): the running max is raised only when a tile's max exceeds it by
-// more than 8; smaller increases are absorbed in p <= 2^8, so O is rescaled rarely.
-// Each score costs one FFMA and one ex2.approx; the sum l is kept in fp32.
+// Softmax (base 2): a running max is raised only when a tile's max exceeds it by more
+// than 8; smaller increases are absorbed in p <= 2^8, so O is rescaled rarely.  Each
+// score costs one FFMA and one ex2.approx; the sums are kept in fp32.
 // Every wait is bounded; on timeout the CTA records GB_ERR_TIMEOUT, every role stops
-// issuing, waits (bounded) for its own outstanding copies and MMAs, the tensor
-// memory is freed and the CTA leaves.
+// issuing, waits (bounded) for its own outstanding copies and MMAs, the tensor memory is
+// freed and the CTA leaves.
 #include <cuda.h>
 
 #include "internal.cuh"
@@ -47,28 +50,33 @@ namespace gb {
 namespace {
 
 constexpr int kRows = 128;     // query rows per tile (MMA M)
-constexpr int kTok = 64;       // tokens per K/V tile (MMA N of Q.K^T, K of P.V)
-constexpr int kStages = 5;
-constexpr int kThreads = 192;
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
-constexpr uint32_t kTmemCols = 256;  // S/P 0: [0, 64), S/P 1: [64, 128), O: [128, 256)
+constexpr int kTok = 128;      // tokens per K/V tile (MMA N of Q.K^T)
+constexpr int kHalf = 64;      // tokens per softmax group (MMA K of one P.V)
+constexpr int kStages = 3;
+constexpr int kThreads = 320;
+constexpr int kProducerWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr uint32_t kTmemCols = 512;  // S/P 0: [0, 128), S/P 1: [128, 256), O_0: [256, 384), O_1: [384, 512)
+constexpr uint32_t kTmemO = 256;
 
-constexpr int kQ = 0;                // 2 buffers x 32 KiB
-constexpr int kKV = 65536;           // kStages x 32 KiB (K 16 KiB + V 16 KiB)
-constexpr int kStage = 32768;
+constexpr int kQ = 0;                // 32 KiB
+constexpr int kKV = 32768;           // kStages x 64 KiB
+constexpr int kStage = 65536;
 constexpr int kBar = kKV + kStages * kStage;  // mbarriers and control words
-constexpr int kSmem = kBar + 256;
+constexpr int kXch = kBar + 256;     // float [2 groups][2 (m, l)][128 rows]
+constexpr int kSmem = kXch + 2048;
 
 // Control area (8-byte mbarriers, then words).
 constexpr int kBarFull = 0;          // [kStages]
 constexpr int kBarEmpty = kBarFull + 8 * kStages;
-constexpr int kBarQFull = kBarEmpty + 8 * kStages;   // [2]
-constexpr int kBarQEmpty = kBarQFull + 16;           // [2]
-constexpr int kBarSFull = kBarQEmpty + 16;           // [2]
+constexpr int kBarQFull = kBarEmpty + 8 * kStages;
+constexpr int kBarQEmpty = kBarQFull + 8;
+constexpr int kBarSFull = kBarQEmpty + 8;            // [2]
 constexpr int kBarPFull = kBarSFull + 16;            // [2]
 constexpr int kBarPvDone = kBarPFull + 16;           // [2]
-constexpr int kWordTmem = kBarPvDone + 16;
+constexpr int kBarXchFull = kBarPvDone + 16;
+constexpr int kBarOFree = kBarXchFull + 8;
+constexpr int kWordTmem = kBarOFree + 8;
 constexpr int kWordAbort = kWordTmem + 4;
 static_assert(kWordAbort + 4 <= 256, "control area");
 static_assert(kSmem <= 232448, "shared memory per block");
@@ -115,12 +123,12 @@ __device__ __forceinline__ void mma_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_
       "r"(tmem_a), "l"(b), "r"(id), "r"(acc));
 }
 
-// One page of one head (K or V) by 4D TMA: coordinates {0, 0, 0, w}, w = first row / 8.
-__device__ __forceinline__ void tma_4d(uint32_t dst, const CUtensorMap* tm, int w, uint32_t bar) {
+// K and V of one page of one head by 5D TMA: coordinates {0, 0, 0, 0, w}, w = first K row / 8.
+__device__ __forceinline__ void tma_page(uint32_t dst, const CUtensorMap* tm, int w, uint32_t bar) {
   asm volatile(
-      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(
+      "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(
           dst),
-      "l"(tm), "r"(0), "r"(0), "r"(0), "r"(w), "r"(bar)
+      "l"(tm), "r"(0), "r"(0), "r"(0), "r"(0), "r"(w), "r"(bar)
       : "memory");
 }
 
@@ -212,7 +220,7 @@ __device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, vol
 template <int G>
 __global__ void __launch_bounds__(kThreads, 1)
     k_grouped(PoolView v, const __grid_constant__ CUtensorMap tm, int layer, const __nv_bfloat16* __restrict__ q,
-              float qscale, long long total_rows) {
+              float qscale, int w_oob) {
   extern __shared__ __align__(1024) unsigned char sm[];
   if (v.ctl[kCtlStepOk] == 0) return;
   const long long units = (long long)v.ctl[kCtlSegTiles] * v.Hkv;
@@ -230,13 +238,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(ctl + kBarFull + 8 * i, 1);
       mbar_init(ctl + kBarEmpty + 8 * i, 1);
     }
+    mbar_init(ctl + kBarQFull, 1);
+    mbar_init(ctl + kBarQEmpty, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(ctl + kBarQFull + 8 * i, 1);
-      mbar_init(ctl + kBarQEmpty + 8 * i, 1);
       mbar_init(ctl + kBarSFull + 8 * i, 1);
-      mbar_init(ctl + kBarPFull + 8 * i, 4);
+      mbar_init(ctl + kBarPFull + 8 * i, 8);
       mbar_init(ctl + kBarPvDone + 8 * i, 1);
     }
+    mbar_init(ctl + kBarXchFull, 8);
+    mbar_init(ctl + kBarOFree, 8);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -255,34 +265,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------------ producer
     if (lane == 0) asm volatile("prefetch.tensormap [%0];" ::"l"(&tm) : "memory");
-    const int ppt = kTok / v.P;                  // pages per K/V tile (1 to 8)
-    const uint32_t page_bytes = (uint32_t)v.P * 256;  // one page of one head: P rows of 256 bytes
-    const int w_oob = (int)(total_rows / 8);     // first row group past the pool: loads zeros
+    const int ppt = kTok / v.P;                     // pages per tile (2 to 16)
+    const uint32_t page_bytes = (uint32_t)v.P * 512;  // K and V of one page of one head
     uint32_t n = 0;  // tiles issued
     int uidx = 0;    // units started
-    for (long long u = blockIdx.x; u < units && !*abort_flag; u += stride, ++uidx) {
+    bool ok = true;
+    for (long long u = blockIdx.x; u < units && ok && !*abort_flag; u += stride, ++uidx) {
       const Unit x = load_unit(v, u);
-      const int qb = uidx & 1;
-      if (uidx >= 2 && !wait_or_abort(ctl + kBarQEmpty + 8 * qb, ((uidx - 2) >> 1) & 1, abort_flag)) break;
-      // Query rows: row r = (member, query head of this KV head); zero rows past the members.
-      unsigned char* qdst = sm + kQ + qb * 32768;
-#pragma unroll 1
-      for (int r = lane; r < kRows; r += 32) {
-        const int m = x.t * members_per_tile + r / G, gg = r % G;
-        const bool valid = m < x.g;
-        const int b = valid ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
-        const uint4* qrow = reinterpret_cast<const uint4*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
-        uint4 buf[16];
-#pragma unroll
-        for (int c = 0; c < 16; ++c) buf[c] = valid ? qrow[c] : make_uint4(0, 0, 0, 0);
-#pragma unroll
-        for (int c = 0; c < 16; ++c) *reinterpret_cast<uint4*>(qdst + (c >> 3) * 16384 + swz(r, (c & 7) * 8)) = buf[c];
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(ctl + kBarQFull + 8 * qb);
-      // K/V tiles of the unit, one 4D TMA per page for K and one for V.  The page ids of
-      // the next 32 pages are loaded by the 32 lanes at once and handed out by shuffle.
       int page_l = 0;
       for (int j = 0; j < x.ntok; ++j, ++n) {
         const uint32_t st = n % kStages;
@@ -291,12 +280,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int tl = (pb + lane) * v.P;
           page_l = tl < x.Ts ? v.tables[(size_t)x.rep * v.max_pages + x.seg_i0 + (x.tok_base + tl) / v.P] : 0;
         }
-        // Lane c < ppt computes the row groups of page c (K and V) of this tile.
-        int wk = w_oob, wv = w_oob;
+        // Lane c < ppt: row group of page c's K slab (pages past the unit load zeros).
+        int w = w_oob;
         {
-          const int c = lane & 7;
-          const int page_c = __shfl_sync(0xffffffffu, page_l, (pb + c) & 31);
-          const int tl = j * kTok + c * v.P;  // token within the unit
+          const int page_c = __shfl_sync(0xffffffffu, page_l, (pb + (lane & 15)) & 31);
+          const int tl = j * kTok + lane * v.P;  // token within the unit
           if (lane < ppt && tl < x.Ts) {
             int page = page_c;
             if (page < 0 || page >= v.num_pages) {
@@ -304,32 +292,45 @@ __global__ void __launch_bounds__(kThreads, 1)
               page = 0;
             }
             const long long slab = (((long long)layer * v.num_pages + page) * 2) * v.Hkv + x.h;
-            wk = (int)(slab * v.P / 8);
-            wv = (int)((slab + v.Hkv) * v.P / 8);
+            w = (int)(slab * v.P / 8);
           }
         }
-        int ws[16];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          ws[2 * c] = __shfl_sync(0xffffffffu, wk, c);
-          ws[2 * c + 1] = __shfl_sync(0xffffffffu, wv, c);
-        }
-        bool ok = true;
-        if (lane == 0) {
-          if (n >= (uint32_t)kStages) ok = wait_or_abort(ctl + kBarEmpty + 8 * st, ((n / kStages) - 1) & 1, abort_flag);
-          if (ok) {
-            const uint32_t bar = ctl + kBarFull + 8 * st;
-            mbar_arrive_expect_tx(bar, kStage);
-            const uint32_t dst0 = sbase + kKV + st * kStage;
-#pragma unroll
-            for (int c = 0; c < 8; ++c)
-              if (c < ppt) {
-                tma_4d(dst0 + c * page_bytes, &tm, ws[2 * c], bar);
-                tma_4d(dst0 + 16384 + c * page_bytes, &tm, ws[2 * c + 1], bar);
-              }
+        if (lane == 0 && n >= (uint32_t)kStages)
+          ok = wait_or_abort(ctl + kBarEmpty + 8 * st, ((n / kStages) - 1) & 1, abort_flag);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (!ok) break;
+        const uint32_t bar = ctl + kBarFull + 8 * st;
+        if (lane == 0) mbar_arrive_expect_tx(bar, kStage);
+        __syncwarp();
+        // Lane c issues page c: a TMA instruction holds its thread for a while, so the
+        // lanes' copies go out in parallel.
+        if (lane < ppt) tma_page(sbase + kKV + st * kStage + lane * page_bytes, &tm, w, bar);
+        if (j == 0) {
+          // Query rows of the unit (after its first tile's copies are under way): row r =
+          // (member, query head of this KV head); zero rows past the members.  The single
+          // Q buffer is free once the previous unit's last S has completed.
+          if (lane == 0 && uidx >= 1) ok = wait_or_abort(ctl + kBarQEmpty, (uidx - 1) & 1, abort_flag);
+          ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+          if (!ok) {
+            ++n;
+            break;
           }
+#pragma unroll 1
+          for (int r = lane; r < kRows; r += 32) {
+            const int m = x.t * members_per_tile + r / G, gg = r % G;
+            const bool valid = m < x.g;
+            const int b = valid ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
+            const uint4* qrow = reinterpret_cast<const uint4*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
+            uint4 buf[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) buf[c] = valid ? qrow[c] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) *reinterpret_cast<uint4*>(sm + kQ + (c >> 3) * 16384 + swz(r, (c & 7) * 8)) = buf[c];
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(ctl + kBarQFull);
         }
-        if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) break;
       }
     }
     // Drain: copies still in flight land before the CTA leaves (bounded).
@@ -347,27 +348,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     int uidx_s = 0, j_s = 0;
     Unit xs{};
     if (u_s < units) xs = load_unit(v, u_s);
-    // S(n_s) can go when its Q buffer is filled (first tile of a unit), its K/V stage has
-    // landed and P.V(n_s - 2), the last reader of its S/P columns, has been issued (the
-    // tensor core executes one CTA's MMAs in issue order).
+    // S(n_s) can go when the Q buffer holds its unit (first tile), its stage has landed
+    // and P.V(n_s - 2), the last reader of its S/P columns, has been issued.
     auto s_ready = [&]() -> bool {
-      if (j_s == 0 && !mbar_test(ctl + kBarQFull + 8 * (uidx_s & 1), (uidx_s >> 1) & 1)) return false;
+      if (j_s == 0 && !mbar_test(ctl + kBarQFull, uidx_s & 1)) return false;
       if (!mbar_test(ctl + kBarFull + 8 * (n_s % kStages), (n_s / kStages) & 1)) return false;
       return n_pv + 1 >= n_s;
     };
     auto issue_s = [&]() {
       const uint32_t st = n_s % kStages, sb = n_s & 1;
       tc_fence_after();
-      const uint32_t qa = sbase + kQ + (uidx_s & 1) * 32768;
       const uint32_t kb = sbase + kKV + st * kStage;
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
-        const uint64_t a = sdesc(qa + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-        const uint64_t b = sdesc(kb + (kk >> 2) * 1024 + (kk & 3) * 32, 16, 2048);
-        mma(tmem + sb * 64, a, b, ID_S, kk > 0);
+        const uint64_t a = sdesc(sbase + kQ + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
+        const uint64_t b = sdesc(kb + (kk >> 2) * 1024 + (kk & 3) * 32, 16, 4096);
+        mma(tmem + sb * 128, a, b, ID_S, kk > 0);
       }
       mma_commit(ctl + kBarSFull + 8 * sb);
-      if (j_s + 1 == xs.ntok) mma_commit(ctl + kBarQEmpty + 8 * (uidx_s & 1));  // last read of this Q buffer
+      if (j_s + 1 == xs.ntok) mma_commit(ctl + kBarQEmpty);  // last read of the Q buffer for this unit
       ++n_s;
       if (++j_s == xs.ntok) {
         j_s = 0;
@@ -377,10 +376,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     };
     if (lane == 0) {
-      // Poll both queues and issue whichever MMA is ready, so P.V(n) never waits behind
-      // the data of tile n+1 and S(n+1) never waits behind the softmax of tile n.
       long long u_p = blockIdx.x;
-      int j_p = 0;
+      int uidx_p = 0, j_p = 0;
       Unit xp = load_unit(v, u_p);
       uint64_t t_progress = globaltimer_ns();
       uint32_t spins = 0;
@@ -391,20 +388,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           progressed = true;
         }
         const uint32_t pb = n_pv & 1, st = n_pv % kStages;
-        if (n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv >> 1) & 1)) {
+        // P.V(n) needs both groups' P; a unit's first P.V also needs the previous unit's
+        // accumulators read out (o_free), since it overwrites them.
+        if (n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv >> 1) & 1) &&
+            (j_p > 0 || uidx_p == 0 || mbar_test(ctl + kBarOFree, (uidx_p - 1) & 1))) {
           tc_fence_after();
-          const uint32_t vb = sbase + kKV + st * kStage + 16384;
+          const uint32_t vb = sbase + kKV + st * kStage + 2048;
 #pragma unroll
-          for (int kk = 0; kk < kTok / 16; ++kk) {
-            // A = P (bf16 pairs in the S columns, 8 columns per 16 tokens), B = V (MN-major).
-            const uint64_t b = sdesc(vb + kk * 4096, 1024, 2048);
-            mma_ts(tmem + 128, tmem + pb * 64 + kk * 8, b, ID_PV, (j_p > 0 || kk > 0) ? 1u : 0u);
-          }
+          for (int k = 0; k < 2; ++k)
+#pragma unroll
+            for (int kk = 0; kk < kHalf / 16; ++kk) {
+              // A = P_k (bf16 pairs, 8 columns per 16 tokens), B = V tokens [64k + 16kk, +16).
+              const uint64_t b = sdesc(vb + (k * 4 + kk) * 8192, 1024, 4096);
+              mma_ts(tmem + kTmemO + k * 128, tmem + pb * 128 + k * 64 + kk * 8, b, ID_PV,
+                     (j_p > 0 || kk > 0) ? 1u : 0u);
+            }
           mma_commit(ctl + kBarEmpty + 8 * st);
           mma_commit(ctl + kBarPvDone + 8 * pb);
           ++n_pv;
           if (++j_p == xp.ntok) {
             j_p = 0;
+            ++uidx_p;
             u_p += stride;
             if (u_p < units) xp = load_unit(v, u_p);
           }
@@ -430,102 +434,127 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     __syncwarp();
   } else {
-    // ------------------------------------------------------------------ softmax (warps 0-3)
-    const int r = tid;  // query row / TMEM lane
-    const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+    // ------------------------------------------------------------------ softmax (warps 0-7)
+    const int grp = warp >> 2;           // softmax group: tokens [64 grp, 64 grp + 64) of each tile
+    const int r = tid & 127;             // query row / TMEM lane
+    const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+    const uint32_t o_own = tmem + kTmemO + grp * 128 + lane_base;
+    float* xch = reinterpret_cast<float*>(sm + kXch);
     uint32_t n = 0;
+    int uidx = 0;
     bool alive = true;
-    for (long long u = blockIdx.x; u < units && alive; u += stride) {
+    for (long long u = blockIdx.x; u < units && alive; u += stride, ++uidx) {
       const Unit x = load_unit(v, u);
       float m_ref = -INFINITY, l = 0.f;
       for (int j = 0; j < x.ntok; ++j, ++n) {
         const uint32_t sb = n & 1;
-        const uint32_t sp_addr = tmem + sb * 64 + lane_base;
+        const uint32_t sp_addr = tmem + sb * 128 + grp * 64 + lane_base;
         if (!wait_or_abort(ctl + kBarSFull + 8 * sb, (n >> 1) & 1, abort_flag)) { alive = false; break; }
         tc_fence_after();
-        float sv[kTok];
-        tmem_ld32(sp_addr, sv);
-        tmem_ld32(sp_addr + 32, sv + 32);
-        // Only a unit's last tile can reach past its tokens (the same for every thread).
-        if ((j + 1) * kTok > x.Ts) {
+        const int valid = min(max(x.Ts - j * kTok - grp * kHalf, 0), kHalf);  // this group's tokens in the tile
+        uint32_t pw[kHalf / 2];
+        if (valid == 0) {
 #pragma unroll
-          for (int c = 0; c < kTok; ++c)
-            if (j * kTok + c >= x.Ts) sv[c] = -INFINITY;
-        }
-        // Max on the raw scores; qscale > 0, so it scales to the max in log2 units.
-        float mr0 = sv[0], mr1 = sv[1];
+          for (int i = 0; i < kHalf / 2; ++i) pw[i] = 0u;
+        } else {
+          float sv[kHalf];
+          tmem_ld32(sp_addr, sv);
+          tmem_ld32(sp_addr + 32, sv + 32);
+          if (valid < kHalf) {  // only a unit's last tile reaches past its tokens
 #pragma unroll
-        for (int c = 2; c < kTok; c += 2) {
-          mr0 = fmaxf(mr0, sv[c]);
-          mr1 = fmaxf(mr1, sv[c + 1]);
-        }
-        const float mt = fmaxf(mr0, mr1) * qscale;
-        const bool raise = mt > m_ref + 8.f;
-        if (j > 0 && __any_sync(0xffffffffu, raise)) {
-          // O must hold P.V(n-1) and nothing newer before it is rescaled.
-          if (!wait_or_abort(ctl + kBarPvDone + 8 * ((n - 1) & 1), ((n - 1) >> 1) & 1, abort_flag)) {
-            alive = false;
-            break;
+            for (int c = 0; c < kHalf; ++c)
+              if (c >= valid) sv[c] = -INFINITY;
           }
-          tc_fence_after();
-          const float alpha = raise ? exp2f(m_ref - mt) : 1.f;
+          // Max on the raw scores; qscale > 0, so it scales to the max in log2 units.
+          float mr0 = sv[0], mr1 = sv[1];
+#pragma unroll
+          for (int c = 2; c < kHalf; c += 2) {
+            mr0 = fmaxf(mr0, sv[c]);
+            mr1 = fmaxf(mr1, sv[c + 1]);
+          }
+          const float mt = fmaxf(mr0, mr1) * qscale;
+          const bool raise = mt > m_ref + 8.f;
+          if (j > 0 && __any_sync(0xffffffffu, raise)) {
+            // O_k must hold P.V(n-1) and nothing newer before it is rescaled.
+            if (!wait_or_abort(ctl + kBarPvDone + 8 * ((n - 1) & 1), ((n - 1) >> 1) & 1, abort_flag)) {
+              alive = false;
+              break;
+            }
+            tc_fence_after();
+            const float alpha = raise ? exp2f(m_ref - mt) : 1.f;
 #pragma unroll 1
-          for (int c0 = 0; c0 < 128; c0 += 32) {
-            float o[32];
-            tmem_ld32(tmem + 128 + c0 + lane_base, o);
+            for (int c0 = 0; c0 < 128; c0 += 32) {
+              float o[32];
+              tmem_ld32(o_own + c0, o);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] *= alpha;
-            tmem_st32(tmem + 128 + c0 + lane_base, o);
+              for (int i = 0; i < 32; ++i) o[i] *= alpha;
+              tmem_st32(o_own + c0, o);
+            }
+            if (raise) l *= alpha;
           }
-          if (raise) l *= alpha;
-        }
-        if (raise) m_ref = mt;
-        // P in bf16 pairs over the first 32 columns of this tile's S.
-        const float neg_m = -m_ref;
-        float l0 = 0.f, l1 = 0.f;
-        uint32_t pw[kTok / 2];
+          if (raise) m_ref = mt;
+          const float neg_m = -m_ref;
+          float l0 = 0.f, l1 = 0.f;
 #pragma unroll
-        for (int c = 0; c < kTok; c += 2) {
-          // p = 2^(s * qscale - m); masked scores give 2^-inf = 0.
-          const float p0 = ex2_approx(fmaf(sv[c], qscale, neg_m));
-          const float p1 = ex2_approx(fmaf(sv[c + 1], qscale, neg_m));
-          const __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
-          pw[c / 2] = *reinterpret_cast<const uint32_t*>(&pr);
-          l0 += p0;
-          l1 += p1;
+          for (int c = 0; c < kHalf; c += 2) {
+            // p = 2^(s * qscale - m); masked scores give 2^-inf = 0.
+            const float p0 = ex2_approx(fmaf(sv[c], qscale, neg_m));
+            const float p1 = ex2_approx(fmaf(sv[c + 1], qscale, neg_m));
+            const __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
+            pw[c / 2] = *reinterpret_cast<const uint32_t*>(&pr);
+            l0 += p0;
+            l1 += p1;
+          }
+          l += l0 + l1;
         }
-        l += l0 + l1;
-        tmem_st32u(sp_addr, pw);
+        tmem_st32u(sp_addr, pw);  // P_k over the first 32 of this group's S columns
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(ctl + kBarPFull + 8 * sb);
       }
       if (!alive) break;
-      // O is final once P.V of the unit's last tile has completed.
+      // Unit end: both accumulators are final once P.V of the last tile has completed.
       const uint32_t last = n - 1;
       if (!wait_or_abort(ctl + kBarPvDone + 8 * (last & 1), (last >> 1) & 1, abort_flag)) break;
       tc_fence_after();
+      xch[(grp * 2 + 0) * 128 + r] = m_ref;
+      xch[(grp * 2 + 1) * 128 + r] = l;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ctl + kBarXchFull);
+      if (!wait_or_abort(ctl + kBarXchFull, uidx & 1, abort_flag)) break;
+      const float m_o = xch[((1 - grp) * 2 + 0) * 128 + r], l_o = xch[((1 - grp) * 2 + 1) * 128 + r];
+      const float m0 = grp == 0 ? m_ref : m_o, l0 = grp == 0 ? l : l_o;
+      const float m1 = grp == 0 ? m_o : m_ref, l1 = grp == 0 ? l_o : l;
+      const float mm = fmaxf(m0, m1);
+      const float a0 = m0 == -INFINITY ? 0.f : exp2f(m0 - mm);
+      const float a1 = m1 == -INFINITY ? 0.f : exp2f(m1 - mm);
       const int m = x.t * members_per_tile + r / G, gg = r % G;
       const int bk = m < x.g ? v.seg_members[x.moff + m] : 0;
       const int b = bk / kMaxSegDepth;
       const int r_idx = v.seg_rec_off[bk] + x.sp;
       const bool has = m < x.g && r_idx < kMaxSegRecords;
       float* rec = v.grec + (((size_t)b * kMaxSegRecords + r_idx) * v.Hkv + x.h) * v.record_floats;
+      // Group k writes columns [64k, 64k + 64) of the merged output.
 #pragma unroll 1
-      for (int c0 = 0; c0 < 128; c0 += 32) {  // warp-collective loads: every lane takes part
-        float o[32];
-        tmem_ld32(tmem + 128 + c0 + lane_base, o);
+      for (int c0 = grp * 64; c0 < grp * 64 + 64; c0 += 32) {  // warp-collective loads: every lane takes part
+        float o0[32], o1[32];
+        tmem_ld32(tmem + kTmemO + c0 + lane_base, o0);
+        tmem_ld32(tmem + kTmemO + 128 + c0 + lane_base, o1);
         if (has) {
 #pragma unroll
           for (int i = 0; i < 32; i += 4)
-            *reinterpret_cast<float4*>(rec + gg * 128 + c0 + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
+            *reinterpret_cast<float4*>(rec + gg * 128 + c0 + i) =
+                make_float4(o0[i] * a0 + o1[i] * a1, o0[i + 1] * a0 + o1[i + 1] * a1, o0[i + 2] * a0 + o1[i + 2] * a1,
+                            o0[i + 3] * a0 + o1[i + 3] * a1);
         }
       }
-      if (has) {
-        rec[G * 128 + gg] = m_ref;
-        rec[G * 128 + G + gg] = l;
+      if (has && grp == 0) {
+        rec[G * 128 + gg] = mm;
+        rec[G * 128 + G + gg] = l0 * a0 + l1 * a1;
       }
       tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ctl + kBarOFree);
     }
   }
 
@@ -538,12 +567,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-// 4D tensor map over the whole pool, which is viewed as rows of D = 128 bf16 (256 bytes):
-// dims {64 dims, 8 rows, 2 halves of D, row groups of 8}, strides {256, 128, 2048} bytes,
-// box {64, 8, 2, P / 8} = one page of one head.  The box lands in shared memory as
-// [row group][half][8 rows][64 dims] with the 128-byte swizzle, so in a 64-token tile the
-// 8-row groups of one half of D sit 2048 bytes apart: the K-major B operand of Q.K^T
-// (SBO 2048, half h at +1024 h) and the MN-major B operand of P.V (LBO 1024, SBO 2048).
+// 5D tensor map over the whole pool, which is viewed as rows of D = 128 bf16 (256 bytes):
+// dims {64 dims, 8 rows, 2 halves of D, K|V, row groups of 8}, strides {256, 128,
+// Hkv * P * 256 (K slab to V slab), 2048} bytes, box {64, 8, 2, 2, P / 8} = K and V of
+// one page of one head.  The box lands in shared memory as [row group][K|V][half][8 rows]
+// [64 dims] with the 128-byte swizzle.  The row-group extent ends with the last K slab,
+// so every coordinate in range addresses a real K and V slab.
 bool make_kv_tensor_map(gb_pool* pool) {
   typedef CUresult (*EncodeFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -557,18 +586,19 @@ bool make_kv_tensor_map(gb_pool* pool) {
       return false;
   }
   const PoolView& v = pool->view;
-  if (v.P % 8 != 0 || kTok % v.P != 0) return false;
+  if (v.P % 8 != 0 || kTok % v.P != 0 || kTok / v.P > 16) return false;
   const unsigned long long rows = (unsigned long long)v.layers * v.num_pages * 2 * v.Hkv * v.P;
   if (rows >= (1ull << 31)) return false;
-  cuuint64_t dims[4] = {64, 8, 2, rows / 8};
-  cuuint64_t strides[3] = {256, 128, 2048};
-  cuuint32_t box[4] = {64, 8, 2, (cuuint32_t)(v.P / 8)};
-  cuuint32_t es[4] = {1, 1, 1, 1};
+  cuuint64_t dims[5] = {64, 8, 2, 2, (rows - (unsigned long long)v.Hkv * v.P) / 8};
+  cuuint64_t strides[4] = {256, 128, (cuuint64_t)v.Hkv * v.P * 256, 2048};
+  cuuint32_t box[5] = {64, 8, 2, 2, (cuuint32_t)(v.P / 8)};
+  cuuint32_t es[5] = {1, 1, 1, 1, 1};
   CUtensorMap* m = reinterpret_cast<CUtensorMap*>(pool->tmap);
-  const CUresult r = encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, v.kv, dims, strides, box, es,
+  const CUresult r = encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, v.kv, dims, strides, box, es,
                             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   pool->have_tmap = r == CUDA_SUCCESS;
+  pool->tmap_oob = (int)dims[4];
   return pool->have_tmap;
 }
 
@@ -581,11 +611,10 @@ static cudaError_t launch_grouped_t(gb_pool* pool, int layer, const void* q, flo
     configured = true;
   }
   const PoolView& v = pool->view;
-  const long long rows = (long long)v.layers * v.num_pages * 2 * v.Hkv * v.P;
   const float qscale = scale * 1.4426950408889634f;
   prof_begin(pool, GB_PROF_GROUPED, s);
   k_grouped<G><<<pool->num_sms, kThreads, kSmem, s>>>(v, *reinterpret_cast<const CUtensorMap*>(pool->tmap), layer,
-                                                     static_cast<const __nv_bfloat16*>(q), qscale, rows);
+                                                     static_cast<const __nv_bfloat16*>(q), qscale, pool->tmap_oob);
   prof_end(pool, GB_PROF_GROUPED, s);
   pool->launches += 1;
   return cudaGetLastError();

@@ -191,6 +191,7 @@ struct gb_pool {
   unsigned long long seg_gen = 0;           // segment rebuilds so far
   alignas(64) unsigned char tmap[128];      // CUtensorMap over the KV pool (grouped path)
   bool have_tmap = false;
+  int tmap_oob = 0;                          // first row group past the tensor map (loads zeros)
   std::string last_error;
   unsigned long long launches = 0;          // kernels launched by this pool
   cudaEvent_t prof_start[GB_PROF_SLOTS] = {};  // caller-owned instrumentation events

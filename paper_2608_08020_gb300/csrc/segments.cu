@@ -111,8 +111,9 @@ __global__ void k_seg_members(PoolView v) {
 }
 
 // One CTA: the grouped work list.  Each segment has ceil(g*G/128) query tiles; each
-// tile is split along the segment's tokens into pieces of `split` tokens so that the
-// list has about two units per multiprocessor (and no beam needs more than
+// tile is split along the segment's tokens into pieces of `split` tokens (a multiple of
+// the grouped kernel's 128-token K/V tile) so that the list has about two units per
+// multiprocessor (and no beam needs more than
 // kMaxSegRecords partial records).  Entries are (segment, tile, split); every beam
 // gets the offsets of its records (one per split of each of its segments).
 __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
@@ -135,10 +136,10 @@ __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
   if (threadIdx.x == 0) {
     const long long work = (long long)tiletok * v.Hkv;              // tile-tokens over all heads
     const long long target_units = 2LL * (v.num_sms > 0 ? v.num_sms : 1);
-    int split = (int)(((work + target_units - 1) / target_units + 63) / 64 * 64);
+    int split = (int)(((work + target_units - 1) / target_units + 127) / 128 * 128);
     const int max_tokens = v.max_pages * v.P;
-    const int min_split = ((max_tokens + (kMaxSegRecords - kMaxSegDepth) - 1) / (kMaxSegRecords - kMaxSegDepth) + 63) /
-                          64 * 64;
+    const int min_split = ((max_tokens + (kMaxSegRecords - kMaxSegDepth) - 1) / (kMaxSegRecords - kMaxSegDepth) + 127) /
+                          128 * 128;
     split = max(split, max(128, min_split));
     s_split = split;
     v.ctl[kCtlSegSplit] = split;
