@@ -57,6 +57,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--beams", type=int, default=0, help="override the workload's beam count (smaller profiling cases)")
     ap.add_argument("--context", type=int, default=0, help="override the workload's context length")
+    ap.add_argument("--breakdown", action="store_true",
+                    help="also time the planner, append and combine kernels (extra event records in the step)")
+    ap.add_argument("--eager", action="store_true",
+                    help="launch the timed steps one by one instead of as one captured CUDA graph")
     return ap.parse_args()
 
 
@@ -298,6 +302,11 @@ def run_ours(args) -> None:
             if prof is not None:
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_DECODE, *prof["dec"][l])
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_GROUPED, *prof["gr"][l])
+                if "app" in prof:
+                    B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_APPEND, *prof["app"][l])
+                    B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_COMBINE, *prof["comb"][l])
+                    if l == 0:
+                        B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PLAN, *prof["plan"])
             pool.decode_attention(l, q[l], k[l], v[l], wl.attn_scale, out[l], flags)
         if is_round(i):
             if prof is not None:
@@ -318,25 +327,45 @@ def run_ours(args) -> None:
         return a, b
     timed_rounds = [i for i in range(W, W + K) if is_round(i)]
     profs = {i: {"dec": [ev_pair() for _ in range(NL)], "gr": [ev_pair() for _ in range(NL)]} for i in range(W, W + K)}
+    if args.breakdown:  # every kernel of the step bracketed (the extra event records cost step time)
+        for i in range(W, W + K):
+            profs[i].update({"app": [ev_pair() for _ in range(NL)], "comb": [ev_pair() for _ in range(NL)],
+                             "plan": ev_pair()})
     for i in timed_rounds:
         profs[i]["probe"], profs[i]["prune"] = ev_pair(), ev_pair()
     torch.cuda.synchronize()
     launches0 = B.gb_pool_launch_count(pool.handle)
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    graph = None
+    if not args.eager:
+        # The K timed steps are captured once into a CUDA graph and launched once, so the
+        # host's per-launch cost is out of the step (every kernel still runs, once, with the
+        # arguments of its own step; the library's event records become graph nodes).
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for i in range(W, W + K):
+                step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)], profs[i])
+        torch.cuda.synchronize()
     clocks = ClockSampler(gpu_id_for_smi(local))
     clocks.start()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
-    for i in range(W, W + K):
-        step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)], profs[i])
+    torch.cuda.nvtx.range_push("timed")  # lets a profiler capture exactly the timed steps
+    if graph is not None:
+        graph.replay()
+    else:
+        for i in range(W, W + K):
+            step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)], profs[i])
+    torch.cuda.nvtx.range_pop()
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     clk = clocks.stop()
-    for which in (B.GB_PROF_DECODE, B.GB_PROF_PROBE, B.GB_PROF_PRUNE, B.GB_PROF_GROUPED):
+    for which in (B.GB_PROF_DECODE, B.GB_PROF_PROBE, B.GB_PROF_PRUNE, B.GB_PROF_GROUPED, B.GB_PROF_PLAN,
+                  B.GB_PROF_APPEND, B.GB_PROF_COMBINE):
         B.gb_pool_set_profile_events(pool.handle, which, None, None)
     stats = B.gb_pool_read_step_stats(pool.handle, max_steps=K)  # one record per timed step
     launches = B.gb_pool_launch_count(pool.handle) - launches0
@@ -350,6 +379,16 @@ def run_ours(args) -> None:
         raise RuntimeError(f"device status {status} after the timed steps: the measurement is invalid")
     dec_ms = [a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["dec"]]
     gr_ms = [a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["gr"]]
+    # In-stream duration of every kernel of a decode step (per layer; the planner once per step).
+    step_kernels_us = None
+    if args.breakdown:
+        step_kernels_us = {
+            "plan": statistics.mean(profs[i]["plan"][0].elapsed_time(profs[i]["plan"][1]) for i in range(W, W + K)) * 1e3,
+            "append": statistics.mean(a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["app"]) * 1e3,
+            "grouped": statistics.mean(gr_ms) * 1e3,
+            "decode": statistics.mean(dec_ms) * 1e3,
+            "combine": statistics.mean(a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["comb"]) * 1e3,
+        }
     prune_us = statistics.mean(profs[i]["prune"][0].elapsed_time(profs[i]["prune"][1]) for i in timed_rounds) * 1e3 \
         if timed_rounds else None
     probe_us = statistics.mean(profs[i]["probe"][0].elapsed_time(profs[i]["probe"][1]) for i in timed_rounds) * 1e3 \
@@ -468,6 +507,7 @@ def run_ours(args) -> None:
                        "schedule": f"decode every step; probe + tournament (K={wl.K}, fanout {wl.fanout}) every "
                                    f"{delta} tokens: {len(timed_rounds)} round(s) in the timed window",
                        "path": args.flags, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                       "launch": "eager" if args.eager else "one CUDA graph of the timed steps",
                        "l2": f"inputs larger than L2: {eff_bytes / 2**30:.2f} GiB of per-beam KV reads per step",
                        "tree_build_s": round(t_build, 2)},
             "attention_us": (dec_avg_s + gr_avg_s) * 1e6,
@@ -475,6 +515,7 @@ def run_ours(args) -> None:
             "attention_tbps_note": "every beam's whole context (K and V of all KV heads) per attention time",
             "decode_kernel_us": dec_avg_s * 1e6,
             "grouped_kernel_us": gr_avg_s * 1e6,
+            "step_kernels_us": step_kernels_us,
             "probe_us": probe_us,
             "prune_branch_us": prune_us,
             "kernels": kernels,

@@ -232,15 +232,22 @@ gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_strea
  * events (cudaEvent_t) immediately before and after one kernel of the
  * following calls on this pool, so a caller can time that kernel alone on its
  * own stream: `which` is GB_PROF_DECODE (the split-KV decode kernel of
- * gb_decode_attention), GB_PROF_PROBE (gb_score_probe) or GB_PROF_PRUNE
- * (gb_prune_branch).  Passing NULL events stops recording.  The events stay
- * owned by the caller.
+ * gb_decode_attention), GB_PROF_PROBE (gb_score_probe), GB_PROF_PRUNE
+ * (gb_prune_branch), GB_PROF_GROUPED (the grouped shared-prefix kernel),
+ * GB_PROF_PLAN (the step planner: page allocation and decode plans, layer 0),
+ * GB_PROF_APPEND (the K/V append of a layer) or GB_PROF_COMBINE (the merge of
+ * partial results).  Passing NULL events stops recording.  The events stay
+ * owned by the caller.  Under stream capture the records become external event
+ * nodes of the graph.
  */
 #define GB_PROF_DECODE 0
 #define GB_PROF_PROBE 1
 #define GB_PROF_PRUNE 2
 #define GB_PROF_GROUPED 3
-#define GB_PROF_SLOTS 4
+#define GB_PROF_PLAN 4
+#define GB_PROF_APPEND 5
+#define GB_PROF_COMBINE 6
+#define GB_PROF_SLOTS 7
 gb_status gb_pool_set_profile_events(gb_pool* pool, int which, void* start_event, void* stop_event);
 
 /*

@@ -29,6 +29,7 @@ EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_poo
            "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
            "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
+GB_PROF_PLAN, GB_PROF_APPEND, GB_PROF_COMBINE = 4, 5, 6
 
 
 class GbPoolConfig(ctypes.Structure):

@@ -398,44 +398,115 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 
 // Merge the partial records of each (beam, kv head) into out[b][h*G+g][:]: the split-KV
 // records of the warps that covered the beam's per-beam range and, in mode 1, the grouped
-// records of the beam's shared-prefix segments.
-__global__ void k_combine(PoolView v, int mode, int W, float* __restrict__ out) {
+// records of the beam's shared-prefix segments (the log-sum-exp merge, base 2).
+// One CTA of 128 threads per (beam, kv head), built so that many loads are in flight:
+//   1. the (m, l) pairs of all records go to shared memory in one sweep;
+//   2. warp w takes query heads g = w, w + 4: M_g = max m, the scale factors
+//      2^(m - M_g) (kept in place of m) and L_g = sum l * 2^(m - M_g);
+//   3. every thread takes 4 consecutive output elements and sums the records 8 at a
+//      time with float4 loads, then divides by L_g.
+// Beams with more than kCombineCache records take the scale factors from global memory.
+constexpr int kCombineCache = 128;
+
+__global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, float* __restrict__ out) {
+  __shared__ float s_m[kCombineCache * 8], s_l[kCombineCache * 8];
+  __shared__ float s_M[8], s_L[8];
   const int bh = blockIdx.x;
   const int b = bh / v.Hkv, h = bh % v.Hkv;
-  const int G = v.G, D = v.D;
+  const int G = v.G, D = v.D, GD = G * D;
   float* ob = out + ((size_t)b * v.Hq + (size_t)h * G) * D;
   const bool ok = v.ctl[kCtlStepOk] != 0 && v.active[b] != 0;
   const int n = ok ? plan_n(v, mode)[b] : 0;
   const int nseg = (ok && mode == 1 && v.grouped) ? v.seg_nrec[b] : 0;  // grouped records of the beam
   if (n == 0 && nseg == 0) {
-    for (int e = threadIdx.x; e < G * D; e += blockDim.x) ob[e] = 0.f;
+    for (int e = threadIdx.x; e < GD; e += blockDim.x) ob[e] = 0.f;
     return;
   }
   const int Tot = plan_off(v, mode)[v.max_beams];
   const int c = Tot > 0 ? (Tot + W - 1) / W : 1;
   const int off = plan_off(v, mode)[b] + h * n;
-  const int first = off / c, last = n > 0 ? (off + n - 1) / c : first - 1;
+  const int first = off / c, npb = n > 0 ? (off + n - 1) / c - first + 1 : 0;  // per-beam records
+  const int R = npb + nseg;
+  const float* prec = v.partials + (size_t)(first + bh) * v.record_floats;
   const float* grec = v.grec + ((size_t)b * kMaxSegRecords * v.Hkv + h) * v.record_floats;
   const size_t gstride = (size_t)v.Hkv * v.record_floats;
-  for (int e = threadIdx.x; e < G * D; e += blockDim.x) {
-    const int g = e / D;
+  auto rec_at = [&](int r) -> const float* {
+    return r < npb ? prec + (size_t)r * v.record_floats : grec + (size_t)(r - npb) * gstride;
+  };
+  const bool cached = R <= kCombineCache;
+  if (cached) {
+    for (int idx = threadIdx.x; idx < R * G; idx += blockDim.x) {
+      const int r = idx / G, g = idx - r * G;
+      const float* rec = rec_at(r);
+      s_m[r * 8 + g] = rec[GD + g];
+      s_l[r * 8 + g] = rec[GD + G + g];
+    }
+    __syncthreads();
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int g = warp; g < G; g += 4) {
     float M = -INFINITY;
-    for (int w = first; w <= last; ++w) M = fmaxf(M, v.partials[(size_t)(w + bh) * v.record_floats + G * D + g]);
-    for (int k = 0; k < nseg; ++k) M = fmaxf(M, grec[k * gstride + G * D + g]);
-    float l = 0.f, acc = 0.f;
-    for (int w = first; w <= last; ++w) {
-      const float* rec = v.partials + (size_t)(w + bh) * v.record_floats;
-      const float sc = exp2f(rec[G * D + g] - M);
-      l = fmaf(rec[G * D + G + g], sc, l);
-      acc = fmaf(rec[e], sc, acc);
+    for (int r = lane; r < R; r += 32) M = fmaxf(M, cached ? s_m[r * 8 + g] : rec_at(r)[GD + g]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+    float L = 0.f;
+    for (int r = lane; r < R; r += 32) {
+      const float m = cached ? s_m[r * 8 + g] : rec_at(r)[GD + g];
+      const float l = cached ? s_l[r * 8 + g] : rec_at(r)[GD + G + g];
+      const float sc = m == -INFINITY ? 0.f : exp2f(m - M);  // a record that saw no token adds nothing
+      L = fmaf(l, sc, L);
+      if (cached) s_m[r * 8 + g] = sc;
     }
-    for (int k = 0; k < nseg; ++k) {
-      const float* rec = grec + k * gstride;
-      const float sc = exp2f(rec[G * D + g] - M);
-      l = fmaf(rec[G * D + G + g], sc, l);
-      acc = fmaf(rec[e], sc, acc);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+    if (lane == 0) {
+      s_M[g] = M;
+      s_L[g] = L;
     }
-    ob[e] = acc / l;
+  }
+  __syncthreads();
+  const bool vec_out = (reinterpret_cast<uintptr_t>(ob) & 15) == 0;
+  for (int e4 = threadIdx.x; e4 < GD / 4; e4 += blockDim.x) {
+    const int g = (e4 * 4) / D;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int r0 = 0; r0 < R; r0 += 8) {
+      float4 x[8];
+      float sc[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int r = r0 + k;
+        if (r < R) {
+          const float* rec = rec_at(r);
+          x[k] = *reinterpret_cast<const float4*>(rec + 4 * e4);
+          if (cached) {
+            sc[k] = s_m[r * 8 + g];
+          } else {
+            const float m = rec[GD + g];
+            sc[k] = m == -INFINITY ? 0.f : exp2f(m - s_M[g]);
+          }
+        } else {
+          x[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+          sc[k] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        acc.x = fmaf(x[k].x, sc[k], acc.x);
+        acc.y = fmaf(x[k].y, sc[k], acc.y);
+        acc.z = fmaf(x[k].z, sc[k], acc.z);
+        acc.w = fmaf(x[k].w, sc[k], acc.w);
+      }
+    }
+    const float L = s_L[g];
+    const float4 res = make_float4(acc.x / L, acc.y / L, acc.z / L, acc.w / L);
+    if (vec_out) {
+      *reinterpret_cast<float4*>(ob + 4 * e4) = res;
+    } else {
+      ob[4 * e4] = res.x;
+      ob[4 * e4 + 1] = res.y;
+      ob[4 * e4 + 2] = res.z;
+      ob[4 * e4 + 3] = res.w;
+    }
   }
 }
 
@@ -456,7 +527,9 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
   prof_end(pool, GB_PROF_DECODE, s);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  prof_begin(pool, GB_PROF_COMBINE, s);
   k_combine<<<pool->view.max_beams * pool->view.Hkv, 128, 0, s>>>(pool->view, mode, W, out);
+  prof_end(pool, GB_PROF_COMBINE, s);
   pool->launches += 2;
   return cudaGetLastError();
 }

@@ -260,6 +260,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(sm + kBar + kWordTmem);
   const long long stride = gridDim.x;
+  // Units go to CTAs in snake order over the work list (sorted longest first): the k-th
+  // unit of CTA c is k * grid + c for even k and k * grid + grid - 1 - c for odd k.
+  auto unit_at = [&](int k) -> long long {
+    return (long long)k * stride + ((k & 1) ? stride - 1 - blockIdx.x : blockIdx.x);
+  };
   constexpr int members_per_tile = kRows / G;
 
   if (warp == kProducerWarp) {
@@ -270,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t n = 0;  // tiles issued
     int uidx = 0;    // units started
     bool ok = true;
-    for (long long u = blockIdx.x; u < units && ok && !*abort_flag; u += stride, ++uidx) {
+    for (long long u = unit_at(0); u < units && ok && !*abort_flag; u = unit_at(++uidx)) {
       const Unit x = load_unit(v, u);
       int page_l = 0;
       for (int j = 0; j < x.ntok; ++j, ++n) {
@@ -344,7 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t ID_PV = idesc(128, true);
     uint32_t n_s = 0, n_pv = 0;  // S and P.V tiles issued
     bool alive = true;
-    long long u_s = blockIdx.x;  // the tile of the next S: unit, unit index, tile in unit
+    long long u_s = unit_at(0);  // the tile of the next S: unit, unit index, tile in unit
     int uidx_s = 0, j_s = 0;
     Unit xs{};
     if (u_s < units) xs = load_unit(v, u_s);
@@ -370,13 +375,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       ++n_s;
       if (++j_s == xs.ntok) {
         j_s = 0;
-        ++uidx_s;
-        u_s += stride;
+        u_s = unit_at(++uidx_s);
         if (u_s < units) xs = load_unit(v, u_s);
       }
     };
     if (lane == 0) {
-      long long u_p = blockIdx.x;
+      long long u_p = unit_at(0);
       int uidx_p = 0, j_p = 0;
       Unit xp = load_unit(v, u_p);
       uint64_t t_progress = globaltimer_ns();
@@ -408,8 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++n_pv;
           if (++j_p == xp.ntok) {
             j_p = 0;
-            ++uidx_p;
-            u_p += stride;
+            u_p = unit_at(++uidx_p);
             if (u_p < units) xp = load_unit(v, u_p);
           }
           progressed = true;
@@ -443,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t n = 0;
     int uidx = 0;
     bool alive = true;
-    for (long long u = blockIdx.x; u < units && alive; u += stride, ++uidx) {
+    for (long long u = unit_at(0); u < units && alive; u = unit_at(++uidx)) {
       const Unit x = load_unit(v, u);
       float m_ref = -INFINITY, l = 0.f;
       for (int j = 0; j < x.ntok; ++j, ++n) {

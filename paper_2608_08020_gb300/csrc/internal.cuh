@@ -201,14 +201,22 @@ struct gb_pool {
 namespace gb {
 gb_status fail(gb_pool* pool, gb_status code, const char* what);
 
-// Instrumentation: record the caller's event pair around one kernel, if set.
+// Instrumentation: record the caller's event pair around one kernel, if set.  Under
+// stream capture the records become external event nodes, so the events are recorded
+// (and can be timed) each time the graph runs.
+inline void prof_record(cudaEvent_t e, cudaStream_t s) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaStreamIsCapturing(s, &cs);
+  cudaEventRecordWithFlags(e, s, cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault);
+}
 inline void prof_begin(gb_pool* p, int which, cudaStream_t s) {
-  if (p->prof_start[which]) cudaEventRecord(p->prof_start[which], s);
+  if (p->prof_start[which]) prof_record(p->prof_start[which], s);
 }
 inline void prof_end(gb_pool* p, int which, cudaStream_t s) {
-  if (p->prof_stop[which]) cudaEventRecord(p->prof_stop[which], s);
+  if (p->prof_stop[which]) prof_record(p->prof_stop[which], s);
 }
 gb_status check_launch(gb_pool* pool, const char* what);
+
 
 // Kernel launchers implemented in the other translation units.
 cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,

@@ -583,7 +583,9 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
     return fail(pool, GB_ERR_INVALID, "append: bad arguments");
   if (layer != pool->next_layer) return fail(pool, GB_ERR_STATE, "layers of a step must be called in order");
   if (layer == 0) {
+    prof_begin(pool, GB_PROF_PLAN, s);
     k_step_begin<<<1, 1024, 0, s>>>(pool->view, n_tokens, pool->view.grouped ? pool->view.seg_cover : nullptr);
+    prof_end(pool, GB_PROF_PLAN, s);
     pool->launches += 1;
     gb_status st = check_launch(pool, "step_begin");
     if (st != GB_OK) return st;
@@ -594,8 +596,10 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
   const long long vecs = 2LL * n_tokens * pool->cfg.max_beams * pool->cfg.num_kv_heads *
                          (pool->view.D * pool->view.esize / 16);
   const int grid = (int)std::min<long long>((vecs + 255) / 256, pool->num_sms * 8LL);
+  prof_begin(pool, GB_PROF_APPEND, s);
   k_append<<<std::max(grid, 1), 256, 0, s>>>(pool->view, layer, n_tokens, static_cast<const char*>(k),
                                              static_cast<const char*>(v));
+  prof_end(pool, GB_PROF_APPEND, s);
   pool->launches += 1;
   gb_status st = check_launch(pool, "append");
   if (st != GB_OK) return st;

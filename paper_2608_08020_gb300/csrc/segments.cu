@@ -22,6 +22,8 @@
 
 namespace gb {
 
+constexpr int kSegLenBuckets = 256;  // work-list entries sorted by length in 128-token tiles (longer ones share the last bucket)
+
 __global__ void k_seg_scan(PoolView v, unsigned long long gen) {
   const int lane = threadIdx.x & 31;
   const int b = (int)((blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5);
@@ -118,7 +120,8 @@ __global__ void k_seg_members(PoolView v) {
 // gets the offsets of its records (one per split of each of its segments).
 __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
   __shared__ int tmp[33];
-  __shared__ int s_split;
+  __shared__ int s_split, s_total;
+  __shared__ int hist[kSegLenBuckets];
   const int nseg = v.ctl[kCtlSegCount];
   const int rows_per_tile = 128;
   const int cap = v.max_beams * kMaxSegRecords;
@@ -148,24 +151,49 @@ __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
   }
   __syncthreads();
   const int split = s_split;
-  int carry = 0;
-  for (int base = 0; base < nseg; base += blockDim.x) {
-    const int s = base + threadIdx.x;
-    const int tiles = s < nseg ? (v.seg_g[s] * v.G + rows_per_tile - 1) / rows_per_tile : 0;
-    const int splits = s < nseg ? (v.seg_len[s] * v.P + split - 1) / split : 0;
-    if (s < nseg) v.seg_splits[s] = splits;
-    int total;
-    const int off = carry + block_exclusive_scan(tiles * splits, tmp, &total);
-    for (int t = 0; t < tiles; ++t)
-      for (int sp = 0; sp < splits; ++sp) {
-        const int e = off + t * splits + sp;
+  // Entries sorted by length (tiles of 128 tokens), longest first, so that the grouped
+  // kernel's snake assignment of units to CTAs balances the work: count entries per
+  // length, lay the lengths out in descending order, then scatter.
+  const int full_len = split / 128;
+  for (int i = threadIdx.x; i < kSegLenBuckets; i += blockDim.x) hist[i] = 0;
+  __syncthreads();
+  for (int sidx = threadIdx.x; sidx < nseg; sidx += blockDim.x) {
+    const int tiles = (v.seg_g[sidx] * v.G + rows_per_tile - 1) / rows_per_tile;
+    const int toks = v.seg_len[sidx] * v.P;
+    const int splits = (toks + split - 1) / split;
+    v.seg_splits[sidx] = splits;
+    const int last_len = min((toks - (splits - 1) * split + 127) / 128, kSegLenBuckets - 1);
+    if (splits > 1) atomicAdd(&hist[min(full_len, kSegLenBuckets - 1)], tiles * (splits - 1));
+    atomicAdd(&hist[last_len], tiles);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int b = kSegLenBuckets - 1; b >= 0; --b) {  // longest first
+      const int c = hist[b];
+      hist[b] = acc;
+      acc += c;
+    }
+    s_total = acc;
+  }
+  __syncthreads();
+  const int carry = s_total;
+  for (int sidx = threadIdx.x; sidx < nseg; sidx += blockDim.x) {
+    const int tiles = (v.seg_g[sidx] * v.G + rows_per_tile - 1) / rows_per_tile;
+    const int toks = v.seg_len[sidx] * v.P;
+    const int splits = v.seg_splits[sidx];
+    for (int sp = 0; sp < splits; ++sp) {
+      const int len = min((min(toks - sp * split, split) + 127) / 128, kSegLenBuckets - 1);
+      const int e0 = atomicAdd(&hist[len], tiles);
+      for (int t = 0; t < tiles; ++t) {
+        const int e = e0 + t;
         if (e < cap) {
-          v.seg_tile_seg[e] = s;
+          v.seg_tile_seg[e] = sidx;
           v.seg_tile_t[e] = t;
           v.seg_tile_split[e] = sp;
         }
       }
-    carry += total;
+    }
   }
   __syncthreads();
   // The list holds at most 9 * max_beams + 2 * SMs entries (each beam sits in at most
