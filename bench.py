@@ -42,7 +42,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 
-def parse_args():
+def parse_args(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=0, help="timed decode steps (0: one tournament interval)")
@@ -61,7 +61,7 @@ def parse_args():
                     help="also time the planner, append and combine kernels (extra event records in the step)")
     ap.add_argument("--eager", action="store_true",
                     help="launch the timed steps one by one instead of as one captured CUDA graph")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def selected_workload(args, rank: int = 0):
@@ -168,7 +168,8 @@ def measured_peaks() -> dict:
 # Oracle sample on host cores (cpu_baseline leg and the reference arm).
 # ---------------------------------------------------------------------------
 def _oracle_worker(wl_dict, slot_hist, positions, barrier, out_q):
-    """Spawned process: materialise its beams' KV, then time fp64 decode attention steps."""
+    """Spawned process: for each layer, materialise its beams' KV (untimed), then time fp64 decode
+    attention of every step; reports the timed seconds summed over layers."""
     from oracle.attention import decode_attention
     from oracle.beams import kv_from_history
     from workload import gen
@@ -176,20 +177,20 @@ def _oracle_worker(wl_dict, slot_hist, positions, barrier, out_q):
     wl = Workload(**wl_dict)
     hscale = [gen.head_scales(wl.seed, l, wl.num_kv_heads, *wl.head_scale) for l in range(wl.num_layers)] \
         if wl.head_scale else None
-    kv = {(s, l): kv_from_history(h, wl.seed, l, wl.num_kv_heads, wl.head_dim, wl.kv_dtype,
-                                  hscale[l] if hscale else None)
-          for s, h in slot_hist for l in range(wl.num_layers)}
     barrier.wait()
-    t0 = time.perf_counter()
-    n = 0
-    for pos in positions:
-        for s, _ in slot_hist:
-            for l in range(wl.num_layers):
-                K, V = kv[(s, l)]
+    timed = 0.0
+    for l in range(wl.num_layers):
+        kv = {s: kv_from_history(h, wl.seed, l, wl.num_kv_heads, wl.head_dim, wl.kv_dtype,
+                                 hscale[l] if hscale else None) for s, h in slot_hist}
+        t0 = time.perf_counter()
+        for pos in positions:
+            for s, _ in slot_hist:
+                K, V = kv[s]
                 q = gen.q_rows(wl.seed, l, s, pos, wl.num_q_heads, wl.head_dim, wl.kv_dtype, wl.q_scale)
                 decode_attention(q, K, V, wl.attn_scale)
-            n += 1
-    out_q.put((time.perf_counter() - t0, n))
+        timed += time.perf_counter() - t0
+        del kv
+    out_q.put((timed, len(positions) * len(slot_hist)))
 
 
 def oracle_sample(wl, steps: int, sample_beams: int, workers: int | None = None) -> dict:
@@ -219,9 +220,8 @@ def oracle_sample(wl, steps: int, sample_beams: int, workers: int | None = None)
         p.start()
         procs.append(p)
     barrier.wait()
-    t0 = time.perf_counter()
     results = [out_q.get() for _ in chunks]
-    t_attn = time.perf_counter() - t0
+    t_attn = max(t for t, _ in results)  # the workers run side by side, one per core
     for p in procs:
         p.join()
     # The tournament part of the schedule: one probe over all beams and one tournament round
@@ -240,8 +240,65 @@ def oracle_sample(wl, steps: int, sample_beams: int, workers: int | None = None)
 
 
 # ---------------------------------------------------------------------------
+# Several ranks (one replica per GPU): the job's time is the slowest rank's.
+# ---------------------------------------------------------------------------
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The largest of every rank's x, returned on every rank (x itself for one rank)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(world: int, beams: int, steps: int, elapsed_ms: float) -> float:
+    """Whole-job beam-tokens/s: every rank decodes `steps` tokens for its `beams` beams."""
+    return world * beams * steps / (elapsed_ms / 1e3)
+
+
+# ---------------------------------------------------------------------------
 # Our arm.
 # ---------------------------------------------------------------------------
+INPUT_BUDGET_BYTES = 16 * 2**30  # device memory for the pre-generated step inputs
+
+
+def capacity_search(wl, dev) -> dict:
+    """Beams of the workload's full context that a fixed pool holds: with every prefix copied
+    (each beam owns all its pages) and with the method's forks sharing prefixes.  The forked
+    count is found by running the whole schedule (seed 0: probe scores, tournaments, forks) in
+    a pool of the same page count for growing beam counts; pages cover all layers, so one layer
+    decides whether a tree fits."""
+    import torch
+
+    from workload.driver import GpuRun
+    pages = wl.pool_pages()
+    copied = pages // wl.pages_per_beam
+
+    def fits(c: int) -> bool:
+        w1 = dataclasses.replace(wl, num_layers=1, beams=c, K=max(1, round(wl.K * c / wl.beams)), pool_bytes=None,
+                                 num_pages=pages)
+        g = GpuRun(w1, device_gen=True, device=str(dev))
+        g.build(upto=wl.context, final_round=True)
+        ok = g.pool.status() == 0
+        del g
+        torch.cuda.empty_cache()
+        return ok
+
+    lo = wl.beams if fits(wl.beams) else 0   # the configured count (the worst-case bound) must fit
+    hi = 1024                                # the library's slot limit
+    if lo and fits(hi):
+        lo = hi
+    while hi - lo > 1 and lo:
+        mid = (lo + hi) // 2
+        if fits(mid):
+            lo = mid
+        else:
+            hi = mid
+    return {"pool_pages": pages, "pool_bytes": wl.pool_bytes, "copied_beams": copied,
+            "forked_beams_configured": wl.beams, "forked_beams_configured_fit": lo >= wl.beams,
+            "forked_beams_max_seed0": lo}
 def run_ours(args) -> None:
     import torch
     import torch.distributed as dist
@@ -261,14 +318,26 @@ def run_ours(args) -> None:
     wl = selected_workload(args, rank)
     flags = B.GB_PATH_AUTO if args.flags == "auto" else B.GB_PATH_PER_BEAM
     W = args.warmup
-    K = args.steps if args.steps > 0 else wl.interval
-    S = W + (K if args.no_e2e else 2 * K)
     C, Hq, Hkv, D, NL = wl.beams, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.num_layers
+    esz_in = 2 if wl.kv_dtype == "bf16" else 4
+    step_input_bytes = NL * C * (Hq + 2 * Hkv) * D * esz_in
+    if args.steps > 0:
+        K = args.steps
+    elif step_input_bytes * wl.interval > INPUT_BUDGET_BYTES:
+        K = 64                               # pre-generated inputs of a whole interval would not fit beside the pool
+    else:
+        K = wl.interval
+    S = W + (K if args.no_e2e else 2 * K)
     delta = wl.interval
+    capacity = capacity_search(wl, dev) if (wl.pool_bytes is not None and rank == 0) else None
 
-    g = GpuRun(wl, device_gen=True, device=str(dev), max_context=wl.context + S + 1, group_min_beams=args.group_min)
+    # A fixed pool holds the tree up to the workload's context: the steps end there.  Otherwise
+    # the timed window starts at the full context.
+    fixed_pool = wl.pool_bytes is not None
+    g = GpuRun(wl, device_gen=True, device=str(dev), max_context=wl.context + (0 if fixed_pool else S) + 1,
+               group_min_beams=args.group_min)
     t_build = time.perf_counter()
-    g.build(upto=wl.context - W)            # the schedule's rounds up to here, then plain appends
+    g.build(upto=wl.context - (S if fixed_pool else W))  # the schedule's rounds up to here, then plain appends
     torch.cuda.synchronize()
     t_build = time.perf_counter() - t_build
     pos0 = g.pos                             # context before the first (warm-up) step
@@ -369,11 +438,7 @@ def run_ours(args) -> None:
         B.gb_pool_set_profile_events(pool.handle, which, None, None)
     stats = B.gb_pool_read_step_stats(pool.handle, max_steps=K)  # one record per timed step
     launches = B.gb_pool_launch_count(pool.handle) - launches0
-    elapsed_ms = t_start.elapsed_time(t_end)
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(t_start.elapsed_time(t_end), world, dev)
     status = pool.status()
     if status != 0:
         raise RuntimeError(f"device status {status} after the timed steps: the measurement is invalid")
@@ -441,7 +506,7 @@ def run_ours(args) -> None:
                         "peak": peak, "unit": "GB/s", "frac": kg["frac_hbm"], "traffic": captured_traffic("k_grouped", wl.name, args.flags),
                         "bytes_per_launch": gr_bytes, "peak_source": f"{peak_src} hbm_gbs"}
 
-    value = world * C * K / (elapsed_ms / 1e3)
+    value = job_value(world, C, K, elapsed_ms)
     ms_per_step = elapsed_ms / K
 
     # End to end through the C ABI with host buffers: each step's inputs copied in from pinned
@@ -481,12 +546,8 @@ def run_ours(args) -> None:
                     d2h += host.numel() * host.element_size()
         e1.record(stream)
         torch.cuda.synchronize()
-        e_ms = e0.elapsed_time(e1)
-        if world > 1:
-            t = torch.tensor([e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e_ms = float(t.item())
-        e2e = {"value": world * C * K / (e_ms / 1e3), "unit": "beam-tokens/s", "h2d_bytes_per_step": int(h2d // K),
+        e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+        e2e = {"value": job_value(world, C, K, e_ms), "unit": "beam-tokens/s", "h2d_bytes_per_step": int(h2d // K),
                "d2h_bytes_per_step": int(d2h // K), "ms_per_step": e_ms / K}
         status = pool.status()
         if status != 0:
@@ -509,7 +570,9 @@ def run_ours(args) -> None:
                        "path": args.flags, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "launch": "eager" if args.eager else "one CUDA graph of the timed steps",
                        "l2": f"inputs larger than L2: {eff_bytes / 2**30:.2f} GiB of per-beam KV reads per step",
-                       "tree_build_s": round(t_build, 2)},
+                       "tree_build_s": round(t_build, 2),
+                       "window": (f"steps end at the full context {wl.context} (fixed {wl.pool_bytes / 1e9:.0f} GB pool)"
+                                  if fixed_pool else f"steps start at the full context {wl.context}")},
             "attention_us": (dec_avg_s + gr_avg_s) * 1e6,
             "attention_tbps": eff_bytes / (dec_avg_s + gr_avg_s) / 1e12,
             "attention_tbps_note": "every beam's whole context (K and V of all KV heads) per attention time",
@@ -519,6 +582,7 @@ def run_ours(args) -> None:
             "probe_us": probe_us,
             "prune_branch_us": prune_us,
             "kernels": kernels,
+            "capacity": capacity,
             "roofline": roofline,
             "e2e": e2e,
             "gpu_launches": int(launches),
