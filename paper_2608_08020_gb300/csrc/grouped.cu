@@ -16,13 +16,17 @@
 //              over the first 32 of its S columns.  At the end of a unit the two groups
 //              exchange (m, l) through shared memory and each writes half of the merged
 //              unnormalised record (m, l, o) of its row;
-//   warp 8     producer: gathers each unit's query rows into the Q buffer and streams
-//              K/V tiles through a 3-stage ring, one 5D TMA per page (K and V of one
-//              head), issued by several lanes at once;
+//   warp 8     producer: takes the next unit from the grid-wide counter (the work list
+//              is sorted longest first, so this is longest-processing-time-first across
+//              the CTAs), publishes it to the other roles through a 4-slot ring,
+//              gathers the unit's query rows into the Q buffer and streams K/V tiles
+//              through a 3-stage ring, one 5D TMA per page (K and V of one head),
+//              issued by several lanes at once;
 //   warp 9     MMA issuer: polls and issues S(n+1) or P.V(n), whichever is ready first;
 //              P.V takes P straight from tensor memory.
-// Handshakes are mbarriers: full/empty per stage, q_full/q_empty, s_full, p_full and
-// pv_done per double-buffered S/P tile, xch_full and o_free per unit.  An S/P buffer is
+// Handshakes are mbarriers: full/empty per stage, sched_full/sched_empty per unit slot,
+// q_full/q_empty, s_full, p_full and pv_done per double-buffered S/P tile, xch_full and
+// o_free per unit.  The last CTA to finish resets the grid-wide counters.  An S/P buffer is
 // reused by S(n+2) only after P.V(n) has been issued: the tensor core runs a CTA's MMAs
 // in issue order, so P(n) has been read before S(n+2) overwrites it.
 //
@@ -76,7 +80,12 @@ constexpr int kBarPFull = kBarSFull + 16;            // [2]
 constexpr int kBarPvDone = kBarPFull + 16;           // [2]
 constexpr int kBarXchFull = kBarPvDone + 16;
 constexpr int kBarOFree = kBarXchFull + 8;
-constexpr int kWordTmem = kBarOFree + 8;
+constexpr int kSchedSlots = 4;
+constexpr int kBarSchedFull = kBarOFree + 8;                  // [kSchedSlots]
+constexpr int kBarSchedEmpty = kBarSchedFull + 8 * kSchedSlots;  // [kSchedSlots]
+constexpr int kSchedConsumers = 10;  // MMA S side, MMA P.V side, 8 softmax warps
+constexpr int kWordSched = kBarSchedEmpty + 8 * kSchedSlots;  // int [kSchedSlots]: unit id, -1 = no more
+constexpr int kWordTmem = kWordSched + 4 * kSchedSlots;
 constexpr int kWordAbort = kWordTmem + 4;
 static_assert(kWordAbort + 4 <= 256, "control area");
 static_assert(kSmem <= 232448, "shared memory per block");
@@ -224,7 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ __align__(1024) unsigned char sm[];
   if (v.ctl[kCtlStepOk] == 0) return;
   const long long units = (long long)v.ctl[kCtlSegTiles] * v.Hkv;
-  if (blockIdx.x >= units) return;
+  if (units == 0) return;
   if (smem_addr(sm) & 1023) {  // the swizzled layouts need a 1024-byte aligned base
     if (threadIdx.x == 0) set_status(v.ctl, GB_ERR_UNSUPPORTED);
     return;
@@ -247,6 +256,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(ctl + kBarXchFull, 8);
     mbar_init(ctl + kBarOFree, 8);
+    for (int i = 0; i < kSchedSlots; ++i) {
+      mbar_init(ctl + kBarSchedFull + 8 * i, 1);
+      mbar_init(ctl + kBarSchedEmpty + 8 * i, kSchedConsumers);
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -259,12 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *reinterpret_cast<volatile uint32_t*>(sm + kBar + kWordTmem);
-  const long long stride = gridDim.x;
-  // Units go to CTAs in snake order over the work list (sorted longest first): the k-th
-  // unit of CTA c is k * grid + c for even k and k * grid + grid - 1 - c for odd k.
-  auto unit_at = [&](int k) -> long long {
-    return (long long)k * stride + ((k & 1) ? stride - 1 - blockIdx.x : blockIdx.x);
-  };
+  volatile int* sched = reinterpret_cast<volatile int*>(sm + kBar + kWordSched);
   constexpr int members_per_tile = kRows / G;
 
   if (warp == kProducerWarp) {
@@ -275,7 +283,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t n = 0;  // tiles issued
     int uidx = 0;    // units started
     bool ok = true;
-    for (long long u = unit_at(0); u < units && ok && !*abort_flag; u = unit_at(++uidx)) {
+    auto fetch = [&]() -> long long {
+      long long id = 0;
+      if (lane == 0) id = atomicAdd(&v.ctl[kCtlGrpNext], 1);
+      return __shfl_sync(0xffffffffu, id, 0);
+    };
+    long long next = fetch();
+    for (;; ++uidx) {
+      if (!ok || *abort_flag) break;
+      // Publish the unit (or the end, -1) in slot uidx % kSchedSlots once every role has
+      // read the unit that slot held before.
+      const int k = uidx & (kSchedSlots - 1);
+      if (lane == 0 && uidx >= kSchedSlots)
+        ok = wait_or_abort(ctl + kBarSchedEmpty + 8 * k, ((uidx / kSchedSlots) - 1) & 1, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) break;
+      const long long u = next;
+      if (lane == 0) {
+        sched[k] = u < units ? (int)u : -1;
+        mbar_arrive(ctl + kBarSchedFull + 8 * k);
+      }
+      if (u >= units) break;
+      next = fetch();  // the following unit, fetched while this one streams
       const Unit x = load_unit(v, u);
       int page_l = 0;
       for (int j = 0; j < x.ntok; ++j, ++n) {
@@ -349,13 +378,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t ID_PV = idesc(128, true);
     uint32_t n_s = 0, n_pv = 0;  // S and P.V tiles issued
     bool alive = true;
-    long long u_s = unit_at(0);  // the tile of the next S: unit, unit index, tile in unit
-    int uidx_s = 0, j_s = 0;
+    int uidx_s = 0, j_s = 0;     // the tile of the next S: unit index, tile in unit
+    bool have_s = false, done_s = false;
     Unit xs{};
-    if (u_s < units) xs = load_unit(v, u_s);
-    // S(n_s) can go when the Q buffer holds its unit (first tile), its stage has landed
-    // and P.V(n_s - 2), the last reader of its S/P columns, has been issued.
+    // S(n_s) can go when its unit is known, the Q buffer holds that unit (first tile), its
+    // stage has landed and P.V(n_s - 2), the last reader of its S/P columns, has been issued.
     auto s_ready = [&]() -> bool {
+      if (!have_s) {
+        const int k = uidx_s & (kSchedSlots - 1);
+        if (!mbar_test(ctl + kBarSchedFull + 8 * k, (uidx_s / kSchedSlots) & 1)) return false;
+        const int id = sched[k];
+        mbar_arrive(ctl + kBarSchedEmpty + 8 * k);
+        if (id < 0) {
+          done_s = true;
+          return false;
+        }
+        xs = load_unit(v, id);
+        have_s = true;
+        j_s = 0;
+      }
       if (j_s == 0 && !mbar_test(ctl + kBarQFull, uidx_s & 1)) return false;
       if (!mbar_test(ctl + kBarFull + 8 * (n_s % kStages), (n_s / kStages) & 1)) return false;
       return n_pv + 1 >= n_s;
@@ -374,27 +415,38 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (j_s + 1 == xs.ntok) mma_commit(ctl + kBarQEmpty);  // last read of the Q buffer for this unit
       ++n_s;
       if (++j_s == xs.ntok) {
-        j_s = 0;
-        u_s = unit_at(++uidx_s);
-        if (u_s < units) xs = load_unit(v, u_s);
+        ++uidx_s;
+        have_s = false;
       }
     };
     if (lane == 0) {
-      long long u_p = unit_at(0);
-      int uidx_p = 0, j_p = 0;
-      Unit xp = load_unit(v, u_p);
+      int uidx_p = 0, j_p = 0;    // the tile of the next P.V
+      bool have_p = false;
+      Unit xp{};
       uint64_t t_progress = globaltimer_ns();
       uint32_t spins = 0;
-      while (u_p < units) {
+      for (;;) {
         bool progressed = false;
-        if (u_s < units && s_ready()) {
+        if (!done_s && s_ready()) {
           issue_s();
           progressed = true;
+        }
+        if (!have_p) {
+          const int k = uidx_p & (kSchedSlots - 1);
+          if (mbar_test(ctl + kBarSchedFull + 8 * k, (uidx_p / kSchedSlots) & 1)) {
+            const int id = sched[k];
+            mbar_arrive(ctl + kBarSchedEmpty + 8 * k);
+            if (id < 0) break;  // every unit's P.V has been issued
+            xp = load_unit(v, id);
+            have_p = true;
+            j_p = 0;
+            progressed = true;
+          }
         }
         const uint32_t pb = n_pv & 1, st = n_pv % kStages;
         // P.V(n) needs both groups' P; a unit's first P.V also needs the previous unit's
         // accumulators read out (o_free), since it overwrites them.
-        if (n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv >> 1) & 1) &&
+        if (have_p && n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv >> 1) & 1) &&
             (j_p > 0 || uidx_p == 0 || mbar_test(ctl + kBarOFree, (uidx_p - 1) & 1))) {
           tc_fence_after();
           const uint32_t vb = sbase + kKV + st * kStage + 2048;
@@ -411,9 +463,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_commit(ctl + kBarPvDone + 8 * pb);
           ++n_pv;
           if (++j_p == xp.ntok) {
-            j_p = 0;
-            u_p = unit_at(++uidx_p);
-            if (u_p < units) xp = load_unit(v, u_p);
+            ++uidx_p;
+            have_p = false;
           }
           progressed = true;
         }
@@ -446,8 +497,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t n = 0;
     int uidx = 0;
     bool alive = true;
-    for (long long u = unit_at(0); u < units && alive; u = unit_at(++uidx)) {
-      const Unit x = load_unit(v, u);
+    for (;; ++uidx) {
+      const int k = uidx & (kSchedSlots - 1);
+      if (!wait_or_abort(ctl + kBarSchedFull + 8 * k, (uidx / kSchedSlots) & 1, abort_flag)) break;
+      const int id = sched[k];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ctl + kBarSchedEmpty + 8 * k);
+      if (id < 0) break;
+      const Unit x = load_unit(v, id);
       float m_ref = -INFINITY, l = 0.f;
       for (int j = 0; j < x.ntok; ++j, ++n) {
         const uint32_t sb = n & 1;
@@ -566,6 +623,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   if (warp == kMmaWarp) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
+  // The last CTA to finish resets the work counter for the next launch.
+  if (tid == 0) {
+    __threadfence();
+    if (atomicAdd(&v.ctl[kCtlGrpDone], 1) == (int)gridDim.x - 1) {
+      v.ctl[kCtlGrpNext] = 0;
+      v.ctl[kCtlGrpDone] = 0;
+      __threadfence();
+    }
+  }
 }
 
 }  // namespace

@@ -38,6 +38,8 @@ enum Ctl : int {
   kCtlSegTileTok = 11, // sum over segments of (128-row tiles) x tokens
   kCtlSteps = 12,      // steps opened so far (index into the step-stats ring)
   kCtlSegSplit = 13,   // tokens per grouped work unit (segments are split along tokens)
+  kCtlGrpNext = 14,    // next grouped work unit to hand out (reset by the grouped kernel's last CTA)
+  kCtlGrpDone = 15,    // grouped-kernel CTAs finished (reset by the last one)
   kCtlWords = 32
 };
 
