@@ -288,23 +288,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) id = atomicAdd(&v.ctl[kCtlGrpNext], 1);
       return __shfl_sync(0xffffffffu, id, 0);
     };
-    long long next = fetch();
     for (;; ++uidx) {
       if (!ok || *abort_flag) break;
-      // Publish the unit (or the end, -1) in slot uidx % kSchedSlots once every role has
-      // read the unit that slot held before.
+      // The next unit is taken only once this CTA has issued every copy of the previous
+      // one (the producer runs a few tiles ahead of the tensor core), so a unit goes to
+      // the CTA that is about to be free.  It (or the end, -1) is published in slot
+      // uidx % kSchedSlots once every role has read the unit that slot held before.
+      const long long u = fetch();
       const int k = uidx & (kSchedSlots - 1);
       if (lane == 0 && uidx >= kSchedSlots)
         ok = wait_or_abort(ctl + kBarSchedEmpty + 8 * k, ((uidx / kSchedSlots) - 1) & 1, abort_flag);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) break;
-      const long long u = next;
       if (lane == 0) {
         sched[k] = u < units ? (int)u : -1;
         mbar_arrive(ctl + kBarSchedFull + 8 * k);
       }
       if (u >= units) break;
-      next = fetch();  // the following unit, fetched while this one streams
       const Unit x = load_unit(v, u);
       int page_l = 0;
       for (int j = 0; j < x.ntok; ++j, ++n) {
