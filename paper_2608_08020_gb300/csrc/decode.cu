@@ -86,6 +86,19 @@ __device__ __forceinline__ void iter_advance(ChunkIter& it, const int* s_n, cons
   }
 }
 
+// The same, as DPC / 2 pairs of consecutive dims (operands of the paired fp32 FMA).
+template <int DT>
+__device__ __forceinline__ void unpack16x2(const uint4& u, float2* f) {
+  if constexpr (DT == GB_BF16) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) f[k] = make_float2(__uint_as_float(w[k] << 16), __uint_as_float(w[k] & 0xffff0000u));
+  } else {
+    f[0] = make_float2(__uint_as_float(u.x), __uint_as_float(u.y));
+    f[1] = make_float2(__uint_as_float(u.z), __uint_as_float(u.w));
+  }
+}
+
 template <int DT, int G>
 __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     k_decode(PoolView v, int layer, const void* __restrict__ qptr, float qscale, int mode, int W) {
@@ -186,8 +199,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     }
   }
 
-  float qr[G][DPL];
-  float o[G][DPL];
+  constexpr int DP2 = DPL / 2, DC2 = DPC / 2;  // dim pairs per lane / per 16-byte piece
+  float2 qr[G][DP2];   // q (pre-scaled) and the accumulator as pairs of dims: every
+  float2 o[G][DP2];    // multiply-add of Q.K and P.V is one paired fp32 FMA (FFMA2)
   float m_run[G];
   float l_lane[NS];
   int L = 0;
@@ -203,12 +217,12 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         const char* qrow = qbase + ((size_t)(it.b * v.Hq + it.h * G + g) * D) * T::ES;
         const uint4 a = *reinterpret_cast<const uint4*>(qrow + 16 * j);
         const uint4 bq = *reinterpret_cast<const uint4*>(qrow + 128 + 16 * j);
-        unpack16<DT>(a, qr[g]);
-        unpack16<DT>(bq, qr[g] + DPC);
+        unpack16x2<DT>(a, qr[g]);
+        unpack16x2<DT>(bq, qr[g] + DC2);
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) {
-          qr[g][d] *= qscale;
-          o[g][d] = 0.f;
+        for (int d = 0; d < DP2; ++d) {
+          qr[g][d] = make_float2(qr[g][d].x * qscale, qr[g][d].y * qscale);
+          o[g][d] = make_float2(0.f, 0.f);
         }
         m_run[g] = -INFINITY;
       }
@@ -239,15 +253,15 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
       const int t = 4 * i + row;
       const uint4 a = *reinterpret_cast<const uint4*>(Ks + t * T::ROW_BYTES + 16 * j);
       const uint4 bq = *reinterpret_cast<const uint4*>(Ks + t * T::ROW_BYTES + 128 + 16 * j);
-      float kf[DPL];
-      unpack16<DT>(a, kf);
-      unpack16<DT>(bq, kf + DPC);
+      float2 kf[DP2];
+      unpack16x2<DT>(a, kf);
+      unpack16x2<DT>(bq, kf + DC2);
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        float sacc = 0.f;
+        float2 sacc = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) sacc = fmaf(qr[g][d], kf[d], sacc);
-        acc[i * G + g] = sacc;
+        for (int d = 0; d < DP2; ++d) sacc = __ffma2_rn(qr[g][d], kf[d], sacc);
+        acc[i * G + g] = sacc.x + sacc.y;
       }
     }
     // Reduce-scatter over the 8 lanes of the row: 4G -> 2G -> G -> G/2 values.
@@ -301,8 +315,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
       for (int g = 0; g < G; ++g) {
         alpha[g] = exp2f(m_run[g] - m_new[g]);
         m_run[g] = m_new[g];
+        const float2 a2 = make_float2(alpha[g], alpha[g]);
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) o[g][d] *= alpha[g];
+        for (int d = 0; d < DP2; ++d) o[g][d] = __fmul2_rn(o[g][d], a2);
       }
 #pragma unroll
       for (int kk = 0; kk < NS; ++kk) l_lane[kk] *= b0 ? alpha[NS + kk] : alpha[kk];
@@ -324,17 +339,19 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
       for (int g = 0; g < G; ++g) pv[g] = pbuf[t * G + g];
       const uint4 a = *reinterpret_cast<const uint4*>(Vs + t * T::ROW_BYTES + 16 * j);
       const uint4 bq = *reinterpret_cast<const uint4*>(Vs + t * T::ROW_BYTES + 128 + 16 * j);
-      float vf[DPL];
-      unpack16<DT>(a, vf);
-      unpack16<DT>(bq, vf + DPC);
+      float2 vf[DP2];
+      unpack16x2<DT>(a, vf);
+      unpack16x2<DT>(bq, vf + DC2);
       if (partial && tok0 + t >= L) {
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) vf[d] = 0.f;
+        for (int d = 0; d < DP2; ++d) vf[d] = make_float2(0.f, 0.f);
       }
 #pragma unroll
-      for (int g = 0; g < G; ++g)
+      for (int g = 0; g < G; ++g) {
+        const float2 p2 = make_float2(pv[g], pv[g]);
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) o[g][d] = fmaf(pv[g], vf[d], o[g][d]);
+        for (int d = 0; d < DP2; ++d) o[g][d] = __ffma2_rn(p2, vf[d], o[g][d]);
+      }
     }
     __syncwarp();
     // The stage is free again: refill it with the chunk kDecodeStages ahead.
@@ -353,9 +370,11 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 #pragma unroll
       for (int g = 0; g < G; ++g)
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) {
-          o[g][d] += __shfl_xor_sync(0xffffffffu, o[g][d], 8);
-          o[g][d] += __shfl_xor_sync(0xffffffffu, o[g][d], 16);
+        for (int d = 0; d < DP2; ++d) {
+          o[g][d].x += __shfl_xor_sync(0xffffffffu, o[g][d].x, 8);
+          o[g][d].y += __shfl_xor_sync(0xffffffffu, o[g][d].y, 8);
+          o[g][d].x += __shfl_xor_sync(0xffffffffu, o[g][d].x, 16);
+          o[g][d].y += __shfl_xor_sync(0xffffffffu, o[g][d].y, 16);
         }
       float lsum[NS], lother[NS];
 #pragma unroll
@@ -376,10 +395,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
           float* oa = rec + g * D + DPC * j;
           float* ob = rec + g * D + D / 2 + DPC * j;
 #pragma unroll
-          for (int e = 0; e < DPC; e += 4) {
-            *reinterpret_cast<float4*>(oa + e) = make_float4(o[g][e], o[g][e + 1], o[g][e + 2], o[g][e + 3]);
-            *reinterpret_cast<float4*>(ob + e) =
-                make_float4(o[g][DPC + e], o[g][DPC + e + 1], o[g][DPC + e + 2], o[g][DPC + e + 3]);
+          for (int e = 0; e < DC2; e += 2) {
+            *reinterpret_cast<float4*>(oa + 2 * e) = make_float4(o[g][e].x, o[g][e].y, o[g][e + 1].x, o[g][e + 1].y);
+            *reinterpret_cast<float4*>(ob + 2 * e) =
+                make_float4(o[g][DC2 + e].x, o[g][DC2 + e].y, o[g][DC2 + e + 1].x, o[g][DC2 + e + 1].y);
           }
         }
       }
