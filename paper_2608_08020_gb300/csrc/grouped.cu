@@ -349,17 +349,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             ++n;
             break;
           }
-#pragma unroll 1
-          for (int r = lane; r < kRows; r += 32) {
+          // Lane l takes rows l, l + 32, l + 64, l + 96: their member beams first, then the
+          // rows two at a time (32 loads of 16 bytes in flight per lane).
+          const uint4* qrow[kRows / 32];
+          bool qvalid[kRows / 32];
+#pragma unroll
+          for (int i = 0; i < kRows / 32; ++i) {
+            const int r = lane + 32 * i;
             const int m = x.t * members_per_tile + r / G, gg = r % G;
-            const bool valid = m < x.g;
-            const int b = valid ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
-            const uint4* qrow = reinterpret_cast<const uint4*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
-            uint4 buf[16];
+            qvalid[i] = m < x.g;
+            const int b = qvalid[i] ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
+            qrow[i] = reinterpret_cast<const uint4*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
+          }
 #pragma unroll
-            for (int c = 0; c < 16; ++c) buf[c] = valid ? qrow[c] : make_uint4(0, 0, 0, 0);
+          for (int i0 = 0; i0 < kRows / 32; i0 += 2) {
+            uint4 buf[2][16];
 #pragma unroll
-            for (int c = 0; c < 16; ++c) *reinterpret_cast<uint4*>(sm + kQ + (c >> 3) * 16384 + swz(r, (c & 7) * 8)) = buf[c];
+            for (int ii = 0; ii < 2; ++ii)
+#pragma unroll
+              for (int c = 0; c < 16; ++c) buf[ii][c] = qvalid[i0 + ii] ? qrow[i0 + ii][c] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+            for (int ii = 0; ii < 2; ++ii)
+#pragma unroll
+              for (int c = 0; c < 16; ++c)
+                *reinterpret_cast<uint4*>(sm + kQ + (c >> 3) * 16384 + swz(lane + 32 * (i0 + ii), (c & 7) * 8)) = buf[ii][c];
           }
           fence_proxy_async_smem();
           __syncwarp();
