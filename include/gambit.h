@@ -189,9 +189,10 @@ gb_status gb_push_scores(gb_pool* pool, const float* scores_dev, const uint8_t* 
  * Active slots are ranked by s_bar descending (ties: lower slot first; NaN
  * last).  Eligible parents are active slots with gen >= warmup and, when
  * eligible_dev is given, eligible_dev[slot] != 0.
- *   Case 1 (fewer active slots than max_beams): the top min(vacant, |B|)
- *   eligible beams get one child each, placed in vacant slots ascending.
- *   Case 2 (all slots active): prune the bottom K_eff = min(K, (fanout-1) x
+ *   Case 1 (fewer active slots than the capacity C, see gb_pool_set_capacity;
+ *   default max_beams): the top min(C - active, |B|) eligible beams get one
+ *   child each, placed in vacant slots ascending.
+ *   Case 2 (C slots active): prune the bottom K_eff = min(K, (fanout-1) x
  *   eligible survivors) beams; each of the top eligible survivors gets
  *   fanout-1 children (the last one the remainder), placed in the pruned
  *   slots ascending.  fanout = 2 is Eq. 3 exactly.
@@ -207,6 +208,18 @@ gb_status gb_push_scores(gb_pool* pool, const float* scores_dev, const uint8_t* 
 gb_status gb_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const uint8_t* eligible_dev,
                           int32_t* parent_out_dev, uint8_t* pruned_out_dev, uint32_t* lineage_out_dev,
                           gb_stream_t stream);
+
+/*
+ * The tree's capacity C (Algorithm 1's C; Section 3.2, Tree view): the
+ * tournament takes Case 1 while fewer than C traces are active and Case 2
+ * otherwise, and Case 1 never grows the active set beyond C.  Default and
+ * maximum: max_beams.  A caller that evicts a trace as a ghost (it keeps its
+ * place in the Tree view but no longer runs, Section 3.2) lowers C by one so
+ * that the ghost still counts against the capacity.  Host-side setting, read
+ * by the next gb_prune_branch calls.  Errors: GB_ERR_INVALID unless
+ * 1 <= capacity <= max_beams.
+ */
+gb_status gb_pool_set_capacity(gb_pool* pool, int capacity);
 
 /*
  * Release slots whose traces completed ("move completed traces to F") or

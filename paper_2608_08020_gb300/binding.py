@@ -27,7 +27,7 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
            "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
-           "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_last_error"]
+           "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
 GB_PROF_PLAN, GB_PROF_APPEND, GB_PROF_COMBINE = 4, 5, 6
 
@@ -91,6 +91,7 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_pool_launch_count": [V, P],
         "gb_paged_decode_noalloc": [P, V],
         "gb_pool_read_step_stats": [V, P, I, P, V],
+        "gb_pool_set_capacity": [V, I],
         "gb_last_error": [V],
     }
     for name, args in sig.items():
@@ -182,6 +183,10 @@ def gb_prune_branch(pool: int, K: int, fanout: int, warmup: int = 0, eligible=No
                     pruned_out=None, lineage_out=None, stream=None) -> None:
     _check(pool, load().gb_prune_branch(pool, K, fanout, warmup, ptr(eligible), ptr(parent_out), ptr(pruned_out),
                                         ptr(lineage_out), stream_handle(stream)), "gb_prune_branch")
+
+
+def gb_pool_set_capacity(pool: int, capacity: int) -> None:
+    _check(pool, load().gb_pool_set_capacity(pool, int(capacity)), "gb_pool_set_capacity")
 
 
 def gb_release(pool: int, slots, n: int, stream=None) -> None:

@@ -190,6 +190,7 @@ struct gb_pool {
   int step_tokens;    // tokens reserved by the open step
   bool seeded;
   int group_min;
+  int capacity = 0;   // the tree's capacity C for the tournament (0: max_beams)
   unsigned long long seg_gen = 0;           // segment rebuilds so far
   alignas(64) unsigned char tmap[128];      // CUtensorMap over the KV pool (grouped path)
   bool have_tmap = false;

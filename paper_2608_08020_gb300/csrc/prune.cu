@@ -23,7 +23,7 @@ __device__ __forceinline__ unsigned rank_key(float m) {
   return ~asc;
 }
 
-__global__ void __launch_bounds__(1024) k_prune_branch(PoolView v, int K, int fanout, int warmup,
+__global__ void __launch_bounds__(1024) k_prune_branch(PoolView v, int C, int K, int fanout, int warmup,
                                                         const uint8_t* __restrict__ elig_mask,
                                                         int* __restrict__ parent_out,
                                                         uint8_t* __restrict__ pruned_out,
@@ -38,7 +38,7 @@ __global__ void __launch_bounds__(1024) k_prune_branch(PoolView v, int K, int fa
   __shared__ int tmp[33];
   __shared__ int s_nchild, s_last;
   const int tid = threadIdx.x;
-  const int cap = v.max_beams;
+  const int cap = v.max_beams;  // physical slots; C <= cap is the tree's capacity
 
   // 1. Active slots, eligibility, compaction into sort keys.
   const bool act = tid < cap && v.active[tid] != 0;
@@ -77,21 +77,21 @@ __global__ void __launch_bounds__(1024) k_prune_branch(PoolView v, int K, int fa
 
   // 3. Routing (identical in every CTA).
   int nchild = 0;
-  if (N > 0 && N < cap) {
+  if (N > 0 && N < C) {
     // Case 1 (Eq. 2): top min(C - N, |B|) eligible traces, one child each, into vacant slots.
     const bool f = tid < N && s_elig[ord[tid]];
     int nb;
     const int pb = block_exclusive_scan(f ? 1 : 0, tmp, &nb);
     if (f) blist[pb] = ord[tid];
-    nchild = min(cap - N, nb);
+    nchild = min(C - N, nb);
     const bool vac = tid < cap && !act;
     int nv;
     const int pv = block_exclusive_scan(vac ? 1 : 0, tmp, &nv);
     if (vac && pv < nchild) cslot[pv] = tid;
     __syncthreads();
     if (tid < nchild) cpar[tid] = blist[tid];
-  } else if (N == cap) {
-    // Case 2 (Eq. 3, fan-out f): prune the bottom K_eff, branch the top eligible survivors.
+  } else if (N > 0) {
+    // Case 2 (Eq. 3, fan-out f; N = C): prune the bottom K_eff, branch the top eligible survivors.
     const int Kc = K < 0 ? 0 : (K > N ? N : K);
     const int nsurv = N - Kc;
     const bool f = tid < nsurv && s_elig[ord[tid]];
@@ -165,7 +165,8 @@ cudaError_t launch_prune_branch(gb_pool* pool, int K, int fanout, int warmup, co
                                 int32_t* parent_out, uint8_t* pruned_out, uint32_t* lineage_out, cudaStream_t s) {
   const int grid = pool->view.max_beams < pool->num_sms ? pool->view.max_beams : pool->num_sms;
   prof_begin(pool, GB_PROF_PRUNE, s);
-  k_prune_branch<<<grid, 1024, 0, s>>>(pool->view, K, fanout, warmup, elig, parent_out, pruned_out,
+  const int C = pool->capacity > 0 ? pool->capacity : pool->view.max_beams;
+  k_prune_branch<<<grid, 1024, 0, s>>>(pool->view, C, K, fanout, warmup, elig, parent_out, pruned_out,
                                        reinterpret_cast<unsigned*>(lineage_out));
   prof_end(pool, GB_PROF_PRUNE, s);
   pool->launches += 1;
@@ -175,6 +176,14 @@ cudaError_t launch_prune_branch(gb_pool* pool, int K, int fanout, int warmup, co
 }  // namespace gb
 
 using namespace gb;
+
+extern "C" gb_status gb_pool_set_capacity(gb_pool* pool, int capacity) {
+  if (!pool) return GB_ERR_INVALID;
+  if (capacity < 1 || capacity > pool->cfg.max_beams)
+    return fail(pool, GB_ERR_INVALID, "set_capacity: 1 <= capacity <= max_beams required");
+  pool->capacity = capacity;
+  return GB_OK;
+}
 
 extern "C" gb_status gb_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const uint8_t* eligible_dev,
                                      int32_t* parent_out_dev, uint8_t* pruned_out_dev, uint32_t* lineage_out_dev,

@@ -70,6 +70,9 @@ class BeamPool:
                      stream=None):
         B.gb_prune_branch(self.handle, K, fanout, warmup, eligible, parent_out, pruned_out, lineage_out, stream)
 
+    def set_capacity(self, capacity: int):
+        B.gb_pool_set_capacity(self.handle, capacity)
+
     def release(self, slots, stream=None):
         B.gb_release(self.handle, slots, int(slots.numel()), stream)
 
