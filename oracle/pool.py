@@ -54,6 +54,7 @@ class PoolOracle:
     def __init__(self, num_pages: int, max_beams: int, max_pages_per_beam: int, page_size: int):
         self.num_pages = num_pages
         self.max_beams = max_beams
+        self.capacity = max_beams   # the tree's capacity C for the tournament (Section 3.2: ghosts count)
         self.max_pages = max_pages_per_beam
         self.P = page_size
         self.refcnt = np.zeros(num_pages, dtype=np.int64)
@@ -180,7 +181,7 @@ class PoolOracle:
                      mask: np.ndarray | None = None) -> tuple[TournamentPlan, np.ndarray, np.ndarray]:
         """One tournament round; returns (plan, parent_of, pruned flags)."""
         plan = tournament(self.mean, self.active, self.eligible(warmup, mask),
-                          self.max_beams, K, fanout)
+                          self.capacity, K, fanout)
         was_active = self.active.copy()
         for s, _ in plan.children:          # the slot's old references go first
             for p in self.tables[s]:

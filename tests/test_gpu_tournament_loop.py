@@ -43,3 +43,37 @@ def test_gpu_loop_matches_simulation(cuda, C, K, fanout, warmup):
     assert tree.case2_rounds == ref.case2_rounds
     assert tree.case1_rounds == ref.case1_rounds
     assert pool.status() == 0
+
+
+@pytest.mark.parametrize("C,K,num_pages", [(32, 8, 600), (64, 16, 1400)])
+def test_gpu_loop_with_ghosts_matches_oracle_loop(cuda, C, K, num_pages):
+    """Memory pressure: both evict the same traces as ghosts, make the same tournaments and
+    end with the same pool, bit for bit (tables, refcounts, free pages, means, lineage)."""
+    from oracle.loop import tournament_loop
+    from paper_2608_08020_gb300.pool import BeamPool
+    from paper_2608_08020_gb300.tree import COMPLETED, GHOST, PRUNED, TournamentLoop
+    from tests.parity import assert_pool_equal
+    seed, interval, mean_len, P = 5, 200, 3000, 64
+
+    def drivers():
+        rng = np.random.default_rng(seed)
+        init = rng.integers(mean_len // 2, 3 * mean_len // 2, size=C)
+        return (init, lambda run: np.array([np.float32(rng.random()) for _ in run], dtype=np.float32),
+                lambda ch, plen: np.array([int(p) + int(rng.integers(mean_len // 4, mean_len)) for p in plen]))
+
+    init, score_fn, target_fn = drivers()
+    ref = tournament_loop(C, K, 2, interval, 0, P, num_pages, 2048, 64, init, score_fn, target_fn)
+    assert ref["ghosts"] > 0
+
+    init, score_fn, target_fn = drivers()
+    pool = BeamPool(num_layers=1, num_q_heads=2, num_kv_heads=1, head_dim=64, page_size=P, kv_dtype="f32",
+                    num_pages=num_pages, max_beams=C, max_pages_per_beam=2048)
+    loop = TournamentLoop(pool, C, K, fanout=2, interval=interval, warmup=0, prompt_len=64)
+    loop.seed(init)
+    tree = loop.run(score_fn, target_fn)
+    tree.check()
+    assert loop.evictions == tree.count(GHOST) == ref["ghosts"]
+    assert tree.branches == ref["branches"] and tree.count(PRUNED) == ref["pruned"]
+    assert tree.count(COMPLETED) == ref["completed"] and tree.running() == ref["running"]
+    assert tree.case1_rounds == ref["case1"] and tree.case2_rounds == ref["case2"]
+    assert_pool_equal(pool.read_state(), ref["pool"], P, means="exact")
