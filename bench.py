@@ -57,6 +57,9 @@ def parse_args(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--beams", type=int, default=0, help="override the workload's beam count (smaller profiling cases)")
     ap.add_argument("--context", type=int, default=0, help="override the workload's context length")
+    ap.add_argument("--probe", choices=["linear", "mlp"], default="linear",
+                    help="scorer at the tournament points: the linear probe of the workloads, or the two-layer MLP")
+    ap.add_argument("--mlp-hidden", type=int, default=512, help="hidden width of the two-layer MLP scorer")
     ap.add_argument("--breakdown", action="store_true",
                     help="also time the planner, append and combine kernels (extra event records in the step)")
     ap.add_argument("--eager", action="store_true",
@@ -364,6 +367,15 @@ def run_ours(args) -> None:
         gpu_gen.normal(hs[n], wl.hidden_dtype, 1, C, wl.hidden, [wl.seed, gen.TAG_HIDDEN, (0, 0, 1), pos0 + s + 1])
     out = torch.empty(NL, C, Hq, D, dtype=torch.float32, device=dev)
     pool = g.pool
+    mlp = None
+    if args.probe == "mlp":       # the two-layer MLP scorer, seeded random weights (no trained scorer here)
+        if wl.hidden_dtype != "bf16" or wl.hidden % 64:
+            raise SystemExit("--probe mlp needs bf16 hidden states of a multiple of 64")
+        gen_w = torch.Generator(device=dev).manual_seed(wl.seed + 1)
+        w1 = (torch.randn(args.mlp_hidden, wl.hidden, generator=gen_w, device=dev) / wl.hidden ** 0.5).to(torch.bfloat16)
+        b1 = torch.randn(args.mlp_hidden, generator=gen_w, device=dev) * 0.1
+        w2 = torch.randn(args.mlp_hidden, generator=gen_w, device=dev) / args.mlp_hidden ** 0.5
+        mlp = (w1, b1, w2, 0.0)
     stream = torch.cuda.current_stream()
 
     def step(i, q, k, v, h, prof=None):
@@ -381,7 +393,10 @@ def run_ours(args) -> None:
             if prof is not None:
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PROBE, *prof["probe"])
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PRUNE, *prof["prune"])
-            pool.score_probe(h, wl.hidden_dtype, g.w, wl.bias, None, g.scores)
+            if mlp is None:
+                pool.score_probe(h, wl.hidden_dtype, g.w, wl.bias, None, g.scores)
+            else:
+                pool.score_mlp(h, *mlp, score_out=g.scores)
             pool.prune_branch(wl.K, wl.fanout, wl.warmup, None, g.parent, g.pruned, g.lineage)
 
     for i in range(W):
@@ -569,6 +584,7 @@ def run_ours(args) -> None:
                                    f"{delta} tokens: {len(timed_rounds)} round(s) in the timed window",
                        "path": args.flags, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "launch": "eager" if args.eager else "one CUDA graph of the timed steps",
+                       "probe": args.probe if args.probe == "linear" else f"mlp (hidden {args.mlp_hidden})",
                        "l2": f"inputs larger than L2: {eff_bytes / 2**30:.2f} GiB of per-beam KV reads per step",
                        "tree_build_s": round(t_build, 2),
                        "window": (f"steps end at the full context {wl.context} (fixed {wl.pool_bytes / 1e9:.0f} GB pool)"

@@ -177,6 +177,23 @@ gb_status gb_score_probe(gb_pool* pool, const void* hidden_dev, int hidden_dtype
                          float* score_out_dev, gb_stream_t stream);
 
 /*
+ * The same update with the two-layer MLP scorer (Section 4 evaluates Gambit with
+ * a light-weight 2-layer MLP scorer; Section 3.1 admits any scorer of the
+ * last-layer hidden state): f(h) = sigmoid(w2 . relu(W1 h + b1) + b2).  The
+ * first layer runs on the tensor cores (bf16 in, fp32 accumulate).
+ *   hidden_dev: [max_beams][hidden_dim] bf16, 16-byte aligned; hidden_dim a
+ *               positive multiple of 64
+ *   w1_dev:     [d_h][hidden_dim] bf16, 16-byte aligned
+ *   b1_dev, w2_dev: [d_h] fp32; b2 the output bias
+ *   boundary_mask_dev, score_out_dev: as gb_score_probe
+ * Errors: GB_ERR_INVALID for bad sizes or alignment; GB_ERR_TOO_LARGE when
+ * max_beams x d_h exceeds 5,242,880 (the pool's partial-sum buffer).
+ */
+gb_status gb_score_mlp(gb_pool* pool, const void* hidden_dev, int hidden_dim, const void* w1_dev,
+                       const float* b1_dev, const float* w2_dev, float b2, int d_h,
+                       const uint8_t* boundary_mask_dev, float* score_out_dev, gb_stream_t stream);
+
+/*
  * Running-mean update with scores computed elsewhere (any scorer f_theta,
  * Section 3.1): for masked active slots, n += 1 and s_bar is updated exactly
  * as in gb_score_probe.  scores_dev: [max_beams] fp32; mask as above.

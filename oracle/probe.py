@@ -24,6 +24,14 @@ def probe_score(h: np.ndarray, w: np.ndarray, bias: float) -> np.ndarray:
     return 1.0 / (1.0 + np.exp(-z))
 
 
+def mlp_probe_score(h: np.ndarray, w1: np.ndarray, b1: np.ndarray, w2: np.ndarray, b2: float) -> np.ndarray:
+    """The two-layer MLP scorer sigma(w2 . relu(W1 h + b1) + b2) in fp64 (Section 4 uses a
+    2-layer MLP scorer; ReLU between the layers).  h: [..., H], w1: [d_h, H], b1, w2: [d_h]."""
+    z = h.astype(np.float64) @ w1.astype(np.float64).T + b1.astype(np.float64)
+    y = np.maximum(z, 0.0) @ w2.astype(np.float64) + float(b2)
+    return 1.0 / (1.0 + np.exp(-y))
+
+
 def running_mean_update(mean: np.float32, n: int, x: np.float32) -> tuple[np.float32, int]:
     """One step of s_bar <- s_bar + (x - s_bar)/n with n counting this score.
 

@@ -27,7 +27,7 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
            "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
-           "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_last_error"]
+           "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_score_mlp", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
 GB_PROF_PLAN, GB_PROF_APPEND, GB_PROF_COMBINE = 4, 5, 6
 
@@ -92,6 +92,7 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_paged_decode_noalloc": [P, V],
         "gb_pool_read_step_stats": [V, P, I, P, V],
         "gb_pool_set_capacity": [V, I],
+        "gb_score_mlp": [V, V, I, V, V, V, F, I, V, V, V],
         "gb_last_error": [V],
     }
     for name, args in sig.items():
@@ -173,6 +174,12 @@ def gb_score_probe(pool: int, hidden, hidden_dtype: int, hidden_dim: int, w, bia
                    score_out=None, stream=None) -> None:
     _check(pool, load().gb_score_probe(pool, ptr(hidden), hidden_dtype, hidden_dim, ptr(w), float(bias), ptr(mask),
                                        ptr(score_out), stream_handle(stream)), "gb_score_probe")
+
+
+def gb_score_mlp(pool: int, hidden, hidden_dim: int, w1, b1, w2, b2: float, d_h: int, mask=None, score_out=None,
+                 stream=None) -> None:
+    _check(pool, load().gb_score_mlp(pool, ptr(hidden), hidden_dim, ptr(w1), ptr(b1), ptr(w2), float(b2), d_h,
+                                     ptr(mask), ptr(score_out), stream_handle(stream)), "gb_score_mlp")
 
 
 def gb_push_scores(pool: int, scores, mask=None, stream=None) -> None:

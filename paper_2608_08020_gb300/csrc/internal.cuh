@@ -21,6 +21,7 @@ constexpr int kMaxSegDepth = 16;
 constexpr int kMaxSegRecords = 48;  // grouped partial records per beam (segments x token splits)
 constexpr int kStatsRing = 4096;   // steps kept in the step-stats ring
 constexpr int kStatsWords = 8;   // grouped segments per beam (deeper shared levels use the per-beam path)
+constexpr int kMlpScratchFloats = 320 * 128 * 128;  // K-split partials of the MLP scorer's first layer (20 MiB)
 
 // Control words at the start of the metadata buffer.
 enum Ctl : int {
@@ -52,6 +53,7 @@ struct MetaLayout {
       seg_mem_off, seg_fill, seg_members, seg_tile_seg, seg_tile_t, grec, seg_bid, seg_rec_off, seg_nrec,
       seg_splits, seg_tile_split;
   int words;            // free-bitmap words
+  size_t mlp_scratch;   // MLP scorer partial sums
   int partial_records;  // split-KV partial records
   int record_floats;    // floats per partial record: G*(D+2)
 };
@@ -104,6 +106,7 @@ struct PoolView {
   int* stats;           // [kStatsRing][kStatsWords] work of recent steps (see gb_pool_read_step_stats)
   float* partials;
   int record_floats;
+  float* mlp_scratch;   // [kMlpScratchFloats] K-split partials of the MLP scorer
 };
 
 // Plan arrays: mode 0 = per-beam only, mode 1 = with grouped coverage.
@@ -232,6 +235,8 @@ bool make_kv_tensor_map(gb_pool* pool);
 cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
                          float bias, const uint8_t* mask, float* score_out, const float* scores_in,
                          cudaStream_t s);
+cudaError_t launch_mlp(gb_pool* pool, const void* hidden, int H, const void* w1, const float* b1, const float* w2,
+                       float b2, int dh, const uint8_t* mask, float* score_out, cudaStream_t s);
 cudaError_t launch_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const uint8_t* elig,
                                 int32_t* parent_out, uint8_t* pruned_out, uint32_t* lineage_out,
                                 cudaStream_t s);

@@ -61,6 +61,7 @@ MetaLayout meta_layout(const gb_pool_config& c) {
   m.seg_splits = take(BD * sizeof(int));
   m.seg_tile_split = take(B * kMaxSegRecords * sizeof(int));
   m.stats = take((size_t)kStatsRing * kStatsWords * sizeof(int));
+  m.mlp_scratch = take((size_t)kMlpScratchFloats * sizeof(float));
   m.total = o;
   return m;
 }
@@ -513,6 +514,7 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   v.seg_tile_split = reinterpret_cast<int*>(m + L.seg_tile_split);
   v.num_sms = p->num_sms;
   v.stats = reinterpret_cast<int*>(m + L.stats);
+  v.mlp_scratch = reinterpret_cast<float*>(m + L.mlp_scratch);
   v.group_min = p->group_min;
   // The grouped tensor-core path needs bf16 K/V with D = 128 (kind::f16 MMAs, 128-byte rows)
   // and pages of 8 to 64 tokens that tile a 64-token K/V tile exactly.

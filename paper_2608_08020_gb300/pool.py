@@ -63,6 +63,9 @@ class BeamPool:
     def score_probe(self, hidden, hidden_dtype: str, w, bias=0.0, mask=None, score_out=None, stream=None):
         B.gb_score_probe(self.handle, hidden, _DT[hidden_dtype], hidden.shape[-1], w, bias, mask, score_out, stream)
 
+    def score_mlp(self, hidden, w1, b1, w2, b2=0.0, mask=None, score_out=None, stream=None):
+        B.gb_score_mlp(self.handle, hidden, hidden.shape[-1], w1, b1, w2, b2, w1.shape[0], mask, score_out, stream)
+
     def push_scores(self, scores, mask=None, stream=None):
         B.gb_push_scores(self.handle, scores, mask, stream)
 

@@ -80,3 +80,38 @@ def test_update_rounds_each_operation_in_fp32():
     d = np.float32(x - m)
     q = np.float32(d / np.float32(3))
     assert running_mean_update(m, n, x)[0] == np.float32(m + q)
+
+
+# -- the two-layer MLP scorer ------------------------------------------------------
+def test_mlp_with_zero_first_layer_is_a_constant():
+    from oracle.probe import mlp_probe_score
+    rng = np.random.default_rng(0)
+    h = rng.standard_normal((5, 64))
+    b1 = np.array([0.5, -2.0, 1.5])
+    w2 = np.array([2.0, 7.0, -1.0])
+    got = mlp_probe_score(h, np.zeros((3, 64)), b1, w2, 0.25)
+    want = 1.0 / (1.0 + np.exp(-(0.5 * 2.0 + 0.0 * 7.0 + 1.5 * -1.0 + 0.25)))   # relu(-2) = 0
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-15)
+
+
+def test_mlp_reduces_to_the_linear_probe():
+    """d_h = 1, a bias large enough that relu is the identity, and an output bias that
+    cancels it: sigma(w.h) exactly as the linear probe."""
+    from oracle.probe import mlp_probe_score, probe_score
+    rng = np.random.default_rng(1)
+    h = rng.standard_normal((7, 128))
+    w = rng.standard_normal(128) / 8
+    big = 1000.0
+    got = mlp_probe_score(h, w[None, :], np.array([big]), np.array([1.0]), -big)
+    np.testing.assert_allclose(got, probe_score(h, w, 0.0), rtol=0, atol=1e-12)
+
+
+def test_mlp_relu_pair_gives_the_absolute_value():
+    """Rows w and -w with unit output weights: relu(x) + relu(-x) = |x|."""
+    from oracle.probe import mlp_probe_score
+    rng = np.random.default_rng(2)
+    h = rng.standard_normal((9, 96))
+    w = rng.standard_normal(96) / 10
+    got = mlp_probe_score(h, np.stack([w, -w]), np.zeros(2), np.ones(2), -0.5)
+    want = 1.0 / (1.0 + np.exp(-(np.abs(h @ w) - 0.5)))
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-12)
