@@ -353,6 +353,89 @@ typedef struct {
 } gb_paged_decode_args;
 gb_status gb_paged_decode_noalloc(const gb_paged_decode_args* args, gb_stream_t stream);
 
+/*
+ * Apply a tournament decided on another pool (for example the generator's pool's
+ * gb_prune_branch parent_out) to this pool: every slot s with parent_of[s] >= 0 and
+ * parent_of[s] != s becomes a child of slot parent_of[s] - it drops its own page
+ * references (pages reaching 0 become free), takes the parent's block table (every
+ * page's refcount + 1; nothing is copied), length, s_bar and n, gen = 0 and a new
+ * lineage id (children in ascending slot order).  Other slots are unchanged.
+ * Section 3.1: a branched trace continues from its parent's state via prefix
+ * caching; this keeps a second per-trace cache (the sequence scorer's) in step.
+ *   parent_of_dev: [max_beams] int32 device array; a parent must keep
+ *                  parent_of[parent] = parent (survivors), and be active.
+ * A parent id >= max_beams records GB_ERR_INVALID in the device status.
+ * Errors: GB_ERR_STATE for an unseeded pool or inside an open step.
+ */
+gb_status gb_fork_slots(gb_pool* pool, const int32_t* parent_of_dev, gb_stream_t stream);
+
+/*
+ * The history-aware sequence scorer (Appendix, "Evaluating Search Generalization",
+ * Eq. 4-6), run incrementally: for each trace's step hidden states h_1 .. h_t,
+ *   x_t = GELU(W_in LN(h_t)),  z_1..z_t = SequenceTransformer(x_1..x_t),
+ *   y_t = sigmoid(w_out . LN(z_t) + b_out).
+ * The transformer has L pre-norm layers: causal multi-head attention with rotary
+ * embeddings (pairs (i, i + 64), angle t * 10000^(-i/64)), Hq query heads over Hkv
+ * key/value heads of 128 dims, then a SwiGLU FFN (W_2 (SiLU(W_1 u) * W_3 u)).
+ * LayerNorms have gain and bias, eps 1e-5; GELU is the erf form; d_model = Hq * 128.
+ *
+ * The scorer's key/value cache is a second gb_pool, the step pool, holding one token
+ * per thought step: num_layers = L, num_q_heads = Hq, num_kv_heads = Hkv, head_dim
+ * 128, kv_dtype GB_BF16, max_beams = the generator pool's.  Position 0 of every
+ * trace is the hidden state at the end of the shared prompt (gb_scorer_seed); each
+ * thought boundary adds one position (gb_scorer_step).  Branching and pruning are
+ * mirrored with gb_fork_slots and gb_release on the step pool.  Matrix products run
+ * on the tensor cores (bf16 operands, fp32 accumulation); the residual stream is fp32.
+ *
+ * Weights: one device buffer, 256-byte aligned, holding these tensors at the offsets
+ * gb_scorer_sizes reports (row-major; "f32" fp32, "bf16" bfloat16):
+ *   0 ln_in gain f32[H], 1 ln_in bias f32[H], 2 W_in bf16[d][H],
+ *   per layer l (base 3 + 8 l): ln1 gain f32[d], ln1 bias f32[d],
+ *     W_qkv bf16[(Hq + 2 Hkv) 128][d] (q heads, then k heads, then v heads),
+ *     W_o bf16[d][d], ln2 gain f32[d], ln2 bias f32[d],
+ *     W_13 bf16[2F][d] (the F rows of W_1, then the F rows of W_3), W_2 bf16[d][F],
+ *   then (base 3 + 8 L): ln_out gain f32[d], ln_out bias f32[d], w_out f32[d], b_out f32[1].
+ * Workspace: one device buffer, 256-byte aligned, of the size gb_scorer_sizes reports;
+ * the caller owns both buffers.  Calls using one workspace must be ordered (one stream).
+ */
+typedef struct {
+  int hidden_dim;  /* H: the generator's hidden size (positive multiple of 64) */
+  int ffn_dim;     /* F: SwiGLU inner size (positive multiple of 64) */
+} gb_scorer_config;
+
+/*
+ * Sizes of the weight buffer and the workspace for a step pool, and the byte offset
+ * of each weight tensor (offsets[0 .. *n_offsets), in the order above; offsets may be
+ * NULL, otherwise max_offsets must be >= 3 + 8 L + 4).  Any output may be NULL.
+ * Errors: GB_ERR_UNSUPPORTED for a step pool or sizes the scorer cannot run on (not
+ * bf16 with 128-dim heads, H or F not multiples of 64, more than 64 layers).
+ */
+gb_status gb_scorer_sizes(gb_pool* step_pool, const gb_scorer_config* cfg, size_t* weight_bytes,
+                          size_t* workspace_bytes, size_t* offsets, int max_offsets, int* n_offsets);
+
+/*
+ * Position 0: run the layer stack on h0_dev (bf16 [H], the hidden state at the end of
+ * the prompt) and seed the step pool's slots 0..n_beams-1 with its per-layer keys and
+ * values (gb_pool_seed with a one-token prompt).
+ * Errors: GB_ERR_STATE if the step pool is already seeded, GB_ERR_INVALID for bad
+ * pointers, alignment or count, plus gb_pool_seed's.
+ */
+gb_status gb_scorer_seed(gb_pool* step_pool, const gb_scorer_config* cfg, const void* weights_dev,
+                         void* workspace_dev, const void* h0_dev, int n_beams, gb_stream_t stream);
+
+/*
+ * One thought boundary for every active slot of the step pool: hidden_dev is bf16
+ * [max_beams][H] (16-byte aligned; rows of inactive slots are ignored), the new
+ * position's key/value is appended to each trace's history and
+ *   score_out_dev[s] = y_t (Eq. 6) of slot s, 0 for inactive slots (fp32 [max_beams]).
+ * Feed the scores to the generator pool's running means with gb_push_scores.
+ * Errors: GB_ERR_STATE for an unseeded step pool or an open step; out of pages in
+ * the step pool is reported in its device status (the scores are then invalid).
+ */
+gb_status gb_scorer_step(gb_pool* step_pool, const gb_scorer_config* cfg, const void* weights_dev,
+                         void* workspace_dev, const void* hidden_dev, float* score_out_dev,
+                         gb_stream_t stream);
+
 /* Short description of the pool's last host-side failure ("" if none); static storage. */
 const char* gb_last_error(gb_pool* pool);
 

@@ -183,10 +183,31 @@ class PoolOracle:
         plan = tournament(self.mean, self.active, self.eligible(warmup, mask),
                           self.capacity, K, fanout)
         was_active = self.active.copy()
-        for s, _ in plan.children:          # the slot's old references go first
-            for p in self.tables[s]:
-                self._unref(p)
-        for k, (s, par) in enumerate(plan.children):
+        self._make_children(plan.children)
+        parent_of = np.where(was_active, np.arange(self.max_beams), -1).astype(np.int64)
+        for s, par in plan.children:
+            parent_of[s] = par
+        pruned = np.zeros(self.max_beams, dtype=np.uint8)
+        pruned[plan.pruned] = 1
+        return plan, parent_of, pruned
+
+    def fork_slots(self, parent_of) -> None:
+        """Apply a tournament decided on another pool (its parent_of): every slot s with
+        parent_of[s] >= 0 and != s becomes a child of parent_of[s] (Section 3.1: a branch
+        continues from its parent's cached prefix), in ascending slot order."""
+        children = [(s, int(p)) for s, p in enumerate(parent_of) if p >= 0 and p != s]
+        if any(p >= self.max_beams for _, p in children):
+            self._set_error(ERR_INVALID)
+        self._make_children([(s, p) for s, p in children if p < self.max_beams])
+
+    def _make_children(self, children) -> None:
+        """Each (slot, parent): the slot drops its references and takes the parent's table
+        (no copy), length, mean and step count, gen 0 and a fresh lineage id."""
+        for s, _ in children:               # the slot's old references go first
+            if self.active[s]:
+                for p in self.tables[s]:
+                    self._unref(p)
+        for k, (s, par) in enumerate(children):
             self.tables[s] = list(self.tables[par])
             for p in self.tables[s]:
                 self._ref(p)
@@ -197,13 +218,7 @@ class PoolOracle:
             self.lineage[s] = self.next_lineage + k
             self.active[s] = True
             self.history[s] = [list(r) for r in self.history[par]]
-        self.next_lineage += len(plan.children)
-        parent_of = np.where(was_active, np.arange(self.max_beams), -1).astype(np.int64)
-        for s, par in plan.children:
-            parent_of[s] = par
-        pruned = np.zeros(self.max_beams, dtype=np.uint8)
-        pruned[plan.pruned] = 1
-        return plan, parent_of, pruned
+        self.next_lineage += len(children)
 
     def release(self, slots) -> None:
         """Completed or evicted traces drop their page references."""

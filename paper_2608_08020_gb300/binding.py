@@ -27,7 +27,8 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
            "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
-           "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_score_mlp", "gb_last_error"]
+           "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_score_mlp", "gb_fork_slots", "gb_scorer_sizes", "gb_scorer_seed",
+           "gb_scorer_step", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
 GB_PROF_PLAN, GB_PROF_APPEND, GB_PROF_COMBINE = 4, 5, 6
 
@@ -93,6 +94,10 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_pool_read_step_stats": [V, P, I, P, V],
         "gb_pool_set_capacity": [V, I],
         "gb_score_mlp": [V, V, I, V, V, V, F, I, V, V, V],
+        "gb_fork_slots": [V, V, V],
+        "gb_scorer_sizes": [V, P, P, P, P, I, P],
+        "gb_scorer_seed": [V, P, V, V, V, I, V],
+        "gb_scorer_step": [V, P, V, V, V, V, V],
         "gb_last_error": [V],
     }
     for name, args in sig.items():
@@ -194,6 +199,33 @@ def gb_prune_branch(pool: int, K: int, fanout: int, warmup: int = 0, eligible=No
 
 def gb_pool_set_capacity(pool: int, capacity: int) -> None:
     _check(pool, load().gb_pool_set_capacity(pool, int(capacity)), "gb_pool_set_capacity")
+
+
+class GbScorerConfig(ctypes.Structure):
+    _fields_ = [("hidden_dim", ctypes.c_int), ("ffn_dim", ctypes.c_int)]
+
+
+def gb_fork_slots(pool: int, parent_of, stream=None) -> None:
+    _check(pool, load().gb_fork_slots(pool, ptr(parent_of), stream_handle(stream)), "gb_fork_slots")
+
+
+def gb_scorer_sizes(pool: int, cfg: GbScorerConfig, max_offsets: int = 4096):
+    """(weight_bytes, workspace_bytes, [offset of each weight tensor])."""
+    wb, wsb, n = ctypes.c_size_t(), ctypes.c_size_t(), ctypes.c_int()
+    offs = (ctypes.c_size_t * max_offsets)()
+    _check(pool, load().gb_scorer_sizes(pool, ctypes.byref(cfg), ctypes.byref(wb), ctypes.byref(wsb), offs,
+                                        max_offsets, ctypes.byref(n)), "gb_scorer_sizes")
+    return wb.value, wsb.value, list(offs[: n.value])
+
+
+def gb_scorer_seed(pool: int, cfg: GbScorerConfig, weights, workspace, h0, n_beams: int, stream=None) -> None:
+    _check(pool, load().gb_scorer_seed(pool, ctypes.byref(cfg), ptr(weights), ptr(workspace), ptr(h0), n_beams,
+                                       stream_handle(stream)), "gb_scorer_seed")
+
+
+def gb_scorer_step(pool: int, cfg: GbScorerConfig, weights, workspace, hidden, score_out, stream=None) -> None:
+    _check(pool, load().gb_scorer_step(pool, ctypes.byref(cfg), ptr(weights), ptr(workspace), ptr(hidden),
+                                       ptr(score_out), stream_handle(stream)), "gb_scorer_step")
 
 
 def gb_release(pool: int, slots, n: int, stream=None) -> None:

@@ -235,6 +235,10 @@ bool make_kv_tensor_map(gb_pool* pool);
 cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
                          float bias, const uint8_t* mask, float* score_out, const float* scores_in,
                          cudaStream_t s);
+// Split-K bf16 GEMM on the tensor cores (gemm.cu): P[s][m][n] over k-range s of A[m][k] B[n][k].
+int gemm_splits(int M, int N, int K, int num_sms, size_t max_floats);
+cudaError_t gemm_partials(const void* A, int M, const void* B, int N, int K, int splits, float* P, int* ctl,
+                          cudaStream_t s);
 cudaError_t launch_mlp(gb_pool* pool, const void* hidden, int H, const void* w1, const float* b1, const float* w2,
                        float b2, int dh, const uint8_t* mask, float* score_out, cudaStream_t s);
 cudaError_t launch_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const uint8_t* elig,

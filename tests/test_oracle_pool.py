@@ -134,3 +134,44 @@ def test_branching_leaves_the_parent_unchanged_and_child_matches_parent():
             np.testing.assert_array_equal(decode_attention(q, *run.beam_kv(b, 0), wl.attn_scale), before[b])
     for s, p in plan.children:  # a child queried with its parent's q gives the parent's output
         np.testing.assert_array_equal(decode_attention(q, *run.beam_kv(s, 0), wl.attn_scale), before[p])
+
+
+def test_fork_slots_replays_a_tournament_decided_elsewhere():
+    """A second pool that applies the first pool's parent_of ends in the same page state
+    as the first (same tables up to page renaming is not enough: both allocate alike, so
+    the tables, refcounts and free pages are equal), and a slot whose parent_of is its
+    own slot or -1 is untouched."""
+    import copy
+    for seed in range(6):
+        r = np.random.default_rng(seed)
+        a = PoolOracle(num_pages=400, max_beams=12, max_pages_per_beam=40, page_size=16)
+        a.seed(9, 20)
+        for _ in range(int(r.integers(1, 40))):
+            a.begin_step()
+        b = copy.deepcopy(a)
+        a.mean[:] = r.random(12).astype(np.float32)
+        _, parent_of, _ = a.prune_branch(K=int(r.integers(0, 5)), fanout=int(r.integers(2, 4)))
+        b.fork_slots(parent_of)
+        assert a.tables == b.tables
+        assert np.array_equal(a.refcnt, b.refcnt) and sorted(a._free) == sorted(b._free)
+        assert np.array_equal(a.active, b.active) and np.array_equal(a.seq_len, b.seq_len)
+        assert np.array_equal(a.lineage, b.lineage) and np.array_equal(a.gen, b.gen)
+        b.check_invariants()
+        for _ in range(20):                          # both grow alike afterwards
+            a.begin_step()
+            b.begin_step()
+        assert a.tables == b.tables
+
+
+def test_fork_slots_by_hand():
+    p = PoolOracle(num_pages=50, max_beams=4, max_pages_per_beam=8, page_size=16)
+    p.seed(3, 16)                                   # page 0 shared by slots 0..2, lineages 1..3
+    for _ in range(16):
+        p.begin_step()                              # private pages 1, 2, 3 of slots 0, 1, 2
+    p.fork_slots([0, 0, 2, 2])                      # slot 1 <- slot 0; vacant slot 3 <- slot 2
+    assert p.tables == [[0, 1], [0, 1], [0, 3], [0, 3]]
+    assert list(p.refcnt[:4]) == [4, 2, 0, 2] and p.num_free() == 47
+    assert list(p.lineage) == [1, 4, 3, 5] and list(p.seq_len) == [32] * 4 and list(p.gen) == [16, 0, 16, 0]
+    p.check_invariants()
+    p.fork_slots([-1, 9, -1, -1])                   # a parent out of range is an error, nothing changes
+    assert p.status == ERR_INVALID and p.tables[1] == [0, 1]
