@@ -57,11 +57,18 @@ def parse_args(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--beams", type=int, default=0, help="override the workload's beam count (smaller profiling cases)")
     ap.add_argument("--context", type=int, default=0, help="override the workload's context length")
-    ap.add_argument("--probe", choices=["linear", "mlp"], default="linear",
-                    help="scorer at the tournament points: the linear probe of the workloads, or the two-layer MLP")
+    ap.add_argument("--probe", choices=["linear", "mlp", "seq"], default="linear",
+                    help="scorer at the tournament points: the linear probe of the workloads, the two-layer MLP, "
+                         "or the history-aware sequence scorer")
     ap.add_argument("--mlp-hidden", type=int, default=512, help="hidden width of the two-layer MLP scorer")
+    ap.add_argument("--seq-shape", default="2,4,2,1024",
+                    help="sequence scorer layers,q-heads,kv-heads,ffn (128-dim heads; d_model = q-heads x 128)")
     ap.add_argument("--breakdown", action="store_true",
                     help="also time the planner, append and combine kernels (extra event records in the step)")
+    ap.add_argument("--event-stride", type=int, default=0,
+                    help="bracket the decode and grouped kernels with CUDA events on every n-th timed step "
+                         "(each event record splits the step's chain of dependent launches; 0: about 32 "
+                         "bracketed steps)")
     ap.add_argument("--eager", action="store_true",
                     help="launch the timed steps one by one instead of as one captured CUDA graph")
     return ap.parse_args(argv)
@@ -302,6 +309,33 @@ def capacity_search(wl, dev) -> dict:
     return {"pool_pages": pages, "pool_bytes": wl.pool_bytes, "copied_beams": copied,
             "forked_beams_configured": wl.beams, "forked_beams_configured_fit": lo >= wl.beams,
             "forked_beams_max_seed0": lo}
+def build_seq_scorer(args, wl, g, dev, n_rounds_after: int):
+    """The sequence scorer with seeded random weights and its step pool, seeded with the
+    prompt's final hidden state and stepped once per tournament round already in the tree
+    (hidden states of those rounds; no forks replayed, so every trace holds that many
+    positions).  Returns the SeqScorer with ``history`` = positions per trace."""
+    from paper_2608_08020_gb300.seqscorer import SeqScorer
+    from workload import gen, gpu_gen
+    from workload.scorer_weights import seqscorer_weights
+    import torch
+    if wl.hidden_dtype != "bf16" or wl.hidden % 64:
+        raise SystemExit("--probe seq needs bf16 hidden states of a multiple of 64")
+    n_layers, hq, hkv, ffn = (int(x) for x in args.seq_shape.split(","))
+    w = seqscorer_weights(wl.seed + 2, wl.hidden, hq * 128, ffn, n_layers, hq, hkv)
+    done = [L for L in wl.rounds() if L <= g.pos]
+    sc = SeqScorer(w, hidden_dim=wl.hidden, ffn_dim=ffn, max_beams=wl.beams,
+                   max_steps=len(done) + n_rounds_after + 2, device=dev)
+    h = torch.empty(wl.beams, wl.hidden, dtype=torch.bfloat16, device=dev)
+    gpu_gen.normal(h, "bf16", 1, wl.beams, wl.hidden, [wl.seed, gen.TAG_HIDDEN, (0, 0, 1), wl.prompt_len])
+    sc.seed(h[0].contiguous(), wl.beams)
+    score = torch.empty(wl.beams, dtype=torch.float32, device=dev)
+    for L in done:
+        gpu_gen.normal(h, "bf16", 1, wl.beams, wl.hidden, [wl.seed, gen.TAG_HIDDEN, (0, 0, 1), L])
+        sc.step(h, score)
+    sc.history = 1 + len(done)
+    return sc
+
+
 def run_ours(args) -> None:
     import torch
     import torch.distributed as dist
@@ -376,28 +410,40 @@ def run_ours(args) -> None:
         b1 = torch.randn(args.mlp_hidden, generator=gen_w, device=dev) * 0.1
         w2 = torch.randn(args.mlp_hidden, generator=gen_w, device=dev) / args.mlp_hidden ** 0.5
         mlp = (w1, b1, w2, 0.0)
+    seq = None
+    if args.probe == "seq":       # the sequence scorer, seeded random weights, its own step pool
+        seq = build_seq_scorer(args, wl, g, dev, n_rounds_after=len(round_steps))
     stream = torch.cuda.current_stream()
 
-    def step(i, q, k, v, h, prof=None):
+    def step(i, q, k, v, h, prof=None, o=None):
+        o = out if o is None else o
         for l in range(NL):
             if prof is not None:
-                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_DECODE, *prof["dec"][l])
-                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_GROUPED, *prof["gr"][l])
+                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_DECODE, *(prof["dec"][l] if "dec" in prof else (None, None)))
+                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_GROUPED, *(prof["gr"][l] if "gr" in prof else (None, None)))
                 if "app" in prof:
                     B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_APPEND, *prof["app"][l])
                     B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_COMBINE, *prof["comb"][l])
                     if l == 0:
                         B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PLAN, *prof["plan"])
-            pool.decode_attention(l, q[l], k[l], v[l], wl.attn_scale, out[l], flags)
+            pool.decode_attention(l, q[l], k[l], v[l], wl.attn_scale, o[l], flags)
         if is_round(i):
             if prof is not None:
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PROBE, *prof["probe"])
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PRUNE, *prof["prune"])
-            if mlp is None:
+            if seq is not None:
+                if prof is not None:
+                    B.gb_pool_set_profile_events(seq.pool.handle, B.GB_PROF_PROBE, *prof["probe"])
+                    B.gb_pool_set_profile_events(seq.pool.handle, B.GB_PROF_PRUNE, *prof["fork"])
+                seq.step(h, g.scores)
+                pool.push_scores(g.scores)
+            elif mlp is None:
                 pool.score_probe(h, wl.hidden_dtype, g.w, wl.bias, None, g.scores)
             else:
                 pool.score_mlp(h, *mlp, score_out=g.scores)
             pool.prune_branch(wl.K, wl.fanout, wl.warmup, None, g.parent, g.pruned, g.lineage)
+            if seq is not None:
+                seq.fork(g.parent)
 
     for i in range(W):
         step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)])
@@ -410,15 +456,20 @@ def run_ours(args) -> None:
         b.record(stream)
         return a, b
     timed_rounds = [i for i in range(W, W + K) if is_round(i)]
-    profs = {i: {"dec": [ev_pair() for _ in range(NL)], "gr": [ev_pair() for _ in range(NL)]} for i in range(W, W + K)}
+    stride = 1 if args.breakdown else max(1, args.event_stride if args.event_stride > 0 else K // 32)
+    inst = [i for i in range(W, W + K) if (i - W) % stride == 0]   # steps whose kernels are bracketed
+    profs = {i: {} for i in range(W, W + K)}
+    for i in inst:
+        profs[i].update({"dec": [ev_pair() for _ in range(NL)], "gr": [ev_pair() for _ in range(NL)]})
     if args.breakdown:  # every kernel of the step bracketed (the extra event records cost step time)
-        for i in range(W, W + K):
+        for i in inst:
             profs[i].update({"app": [ev_pair() for _ in range(NL)], "comb": [ev_pair() for _ in range(NL)],
                              "plan": ev_pair()})
     for i in timed_rounds:
-        profs[i]["probe"], profs[i]["prune"] = ev_pair(), ev_pair()
+        profs[i]["probe"], profs[i]["prune"], profs[i]["fork"] = ev_pair(), ev_pair(), ev_pair()
     torch.cuda.synchronize()
     launches0 = B.gb_pool_launch_count(pool.handle)
+    seq_launches0 = B.gb_pool_launch_count(seq.pool.handle) if seq is not None else 0
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     graph = None
     if not args.eager:
@@ -451,28 +502,36 @@ def run_ours(args) -> None:
     for which in (B.GB_PROF_DECODE, B.GB_PROF_PROBE, B.GB_PROF_PRUNE, B.GB_PROF_GROUPED, B.GB_PROF_PLAN,
                   B.GB_PROF_APPEND, B.GB_PROF_COMBINE):
         B.gb_pool_set_profile_events(pool.handle, which, None, None)
+        if seq is not None:
+            B.gb_pool_set_profile_events(seq.pool.handle, which, None, None)
     stats = B.gb_pool_read_step_stats(pool.handle, max_steps=K)  # one record per timed step
     launches = B.gb_pool_launch_count(pool.handle) - launches0
+    if seq is not None:
+        launches += B.gb_pool_launch_count(seq.pool.handle) - seq_launches0
+        if seq.pool.status() != 0:
+            raise RuntimeError("sequence scorer's step pool reported an error: the measurement is invalid")
     elapsed_ms = max_over_ranks(t_start.elapsed_time(t_end), world, dev)
     status = pool.status()
     if status != 0:
         raise RuntimeError(f"device status {status} after the timed steps: the measurement is invalid")
-    dec_ms = [a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["dec"]]
-    gr_ms = [a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["gr"]]
+    dec_ms = [a.elapsed_time(b) for i in inst for a, b in profs[i]["dec"]]
+    gr_ms = [a.elapsed_time(b) for i in inst for a, b in profs[i]["gr"]]
     # In-stream duration of every kernel of a decode step (per layer; the planner once per step).
     step_kernels_us = None
     if args.breakdown:
         step_kernels_us = {
-            "plan": statistics.mean(profs[i]["plan"][0].elapsed_time(profs[i]["plan"][1]) for i in range(W, W + K)) * 1e3,
-            "append": statistics.mean(a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["app"]) * 1e3,
+            "plan": statistics.mean(profs[i]["plan"][0].elapsed_time(profs[i]["plan"][1]) for i in inst) * 1e3,
+            "append": statistics.mean(a.elapsed_time(b) for i in inst for a, b in profs[i]["app"]) * 1e3,
             "grouped": statistics.mean(gr_ms) * 1e3,
             "decode": statistics.mean(dec_ms) * 1e3,
-            "combine": statistics.mean(a.elapsed_time(b) for i in range(W, W + K) for a, b in profs[i]["comb"]) * 1e3,
+            "combine": statistics.mean(a.elapsed_time(b) for i in inst for a, b in profs[i]["comb"]) * 1e3,
         }
     prune_us = statistics.mean(profs[i]["prune"][0].elapsed_time(profs[i]["prune"][1]) for i in timed_rounds) * 1e3 \
         if timed_rounds else None
     probe_us = statistics.mean(profs[i]["probe"][0].elapsed_time(profs[i]["probe"][1]) for i in timed_rounds) * 1e3 \
         if timed_rounds else None
+    fork_us = statistics.mean(profs[i]["fork"][0].elapsed_time(profs[i]["fork"][1]) for i in timed_rounds) * 1e3 \
+        if (timed_rounds and seq is not None) else None
     grouped_on = flags != B.GB_PATH_PER_BEAM and wl.kv_dtype == "bf16" and D == 128
 
     # Algorithmic work per launch, from the library's per-step records:
@@ -483,6 +542,7 @@ def run_ours(args) -> None:
     kv_tok = 2 * Hkv * D * esz
     q_bytes = C * Hq * D * esz
     assert len(stats) == K, (len(stats), K)
+    stats = [stats[i - W] for i in inst]       # the bracketed steps' work, to match their durations
     dec_tokens = [int(s[1] if grouped_on else s[0]) for s in stats]
     dec_bytes = statistics.mean(t * kv_tok + q_bytes for t in dec_tokens)
     eff_bytes = statistics.mean(int(s[0]) * kv_tok + q_bytes for s in stats)   # as if every beam read everything
@@ -528,42 +588,82 @@ def run_ours(args) -> None:
     # memory and its outputs read back, inside the timed region.
     e2e = None
     if not args.no_e2e:
-        sl = slice(W + K, W + 2 * K)
-        hq, hk, hv = (t[sl].cpu().pin_memory() for t in (qs, ks, vs))
+        # End to end: every step's q, k, v (and, at a round, the hidden states) come from
+        # pinned host memory in one copy, and the step's attention output (and, at a round,
+        # the scores and the tournament's outputs) go back to pinned host memory.  Copies
+        # run on a second stream into double buffers, overlapping the previous step.
+        sl = range(W + K, W + 2 * K)
+        parts = (qs, ks, vs)
+        nbytes = [t[0].numel() * t.element_size() for t in parts]
+        offs = [0, nbytes[0], nbytes[0] + nbytes[1]]
+        in_bytes = sum(nbytes)
+        hin = torch.empty((K, in_bytes), dtype=torch.uint8).pin_memory()
+        for n, i in enumerate(sl):
+            for t, o0, nb in zip(parts, offs, nbytes):
+                hin[n, o0:o0 + nb].copy_(t[i].reshape(-1).view(torch.uint8).cpu())
         hh = hs.cpu().pin_memory()
-        q_d, k_d, v_d = (torch.empty_like(t[0]) for t in (qs, ks, vs))
-        h_d = torch.empty_like(hs[0])
-        o_h = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-        s_h = torch.empty(C, dtype=torch.float32).pin_memory()
-        p_h = torch.empty(C, dtype=torch.int32).pin_memory()
-        pr_h = torch.empty(C, dtype=torch.uint8).pin_memory()
-        ln_h = torch.empty(C, dtype=torch.int32).pin_memory()
+        din = [torch.empty(in_bytes, dtype=torch.uint8, device=dev) for _ in range(2)]
+        views = [[din[b][o0:o0 + nb].view(t.dtype).view(t[0].shape) for t, o0, nb in zip(parts, offs, nbytes)]
+                 for b in range(2)]
+        h_d = [torch.empty_like(hs[0]) for _ in range(2)]
+        dout = [torch.empty_like(out) for _ in range(2)]
+        o_h = [torch.empty(out.shape, dtype=out.dtype).pin_memory() for _ in range(2)]
+        r_h = {n: [torch.empty(C, dtype=t.dtype).pin_memory() for t in (g.scores, g.parent, g.pruned, g.lineage)]
+               for n, i in enumerate(sl) if is_round(i)}
+        cs = torch.cuda.Stream(device=dev)
+        ev = lambda: torch.cuda.Event()
+        loaded, done, outfree = ([ev() for _ in range(2)] for _ in range(3))
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         h2d = d2h = 0
+
+        def load(n):                         # inputs of e2e step n into buffer n % 2 (copy stream)
+            nonlocal h2d
+            b = n % 2
+            with torch.cuda.stream(cs):
+                if n >= 2:
+                    cs.wait_event(done[b])
+                din[b].copy_(hin[n], non_blocking=True)
+                h2d += in_bytes
+                if is_round(sl[n]):
+                    h_d[b].copy_(hh[h_index[sl[n]]], non_blocking=True)
+                    h2d += hh[0].numel() * hh.element_size()
+                loaded[b].record(cs)
+
         e0.record(stream)
-        for n, i in enumerate(range(W + K, W + 2 * K)):
-            q_d.copy_(hq[n], non_blocking=True)
-            k_d.copy_(hk[n], non_blocking=True)
-            v_d.copy_(hv[n], non_blocking=True)
-            h2d += sum(t[n].numel() * t.element_size() for t in (hq, hk, hv))
-            if is_round(i):
-                h_d.copy_(hh[h_index[i]], non_blocking=True)
-                h2d += hh[0].numel() * hh.element_size()
-            step(i, q_d, k_d, v_d, h_d)
-            o_h.copy_(out, non_blocking=True)
-            d2h += o_h.numel() * o_h.element_size()
-            if is_round(i):
-                for host, dev_t in ((s_h, g.scores), (p_h, g.parent), (pr_h, g.pruned), (ln_h, g.lineage)):
-                    host.copy_(dev_t, non_blocking=True)
-                    d2h += host.numel() * host.element_size()
+        t_host = time.perf_counter()
+        cs.wait_stream(stream)
+        load(0)
+        for n, i in enumerate(sl):
+            b = n % 2
+            if n + 1 < K:
+                load(n + 1)
+            stream.wait_event(loaded[b])
+            if n >= 2:
+                stream.wait_event(outfree[b])
+            step(i, *views[b], h_d[b], o=dout[b])
+            done[b].record(stream)
+            with torch.cuda.stream(cs):
+                cs.wait_event(done[b])
+                o_h[b].copy_(dout[b], non_blocking=True)
+                d2h += o_h[b].numel() * o_h[b].element_size()
+                if is_round(i):
+                    for host, dev_t in zip(r_h[n], (g.scores, g.parent, g.pruned, g.lineage)):
+                        host.copy_(dev_t, non_blocking=True)
+                        d2h += host.numel() * host.element_size()
+                outfree[b].record(cs)
+        stream.wait_stream(cs)
         e1.record(stream)
+        t_host = time.perf_counter() - t_host
         torch.cuda.synchronize()
         e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
         e2e = {"value": job_value(world, C, K, e_ms), "unit": "beam-tokens/s", "h2d_bytes_per_step": int(h2d // K),
-               "d2h_bytes_per_step": int(d2h // K), "ms_per_step": e_ms / K}
+               "d2h_bytes_per_step": int(d2h // K), "ms_per_step": e_ms / K,
+               "host_issue_us_per_step": t_host / K * 1e6,
+               "path": "eager calls of the pool API; inputs copied from pinned host memory and outputs read back "
+                       "every step, on a copy stream double-buffered against compute"}
         status = pool.status()
         if status != 0:
             raise RuntimeError(f"device status {status} after the e2e steps: the measurement is invalid")
@@ -584,7 +684,12 @@ def run_ours(args) -> None:
                                    f"{delta} tokens: {len(timed_rounds)} round(s) in the timed window",
                        "path": args.flags, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "launch": "eager" if args.eager else "one CUDA graph of the timed steps",
-                       "probe": args.probe if args.probe == "linear" else f"mlp (hidden {args.mlp_hidden})",
+                       "kernel_events": f"decode and grouped kernels bracketed by CUDA events on {len(inst)} of the "
+                                        f"{K} timed steps (every {stride})",
+                       "probe": {"linear": "linear", "mlp": f"mlp (hidden {args.mlp_hidden})",
+                                 "seq": f"sequence scorer (layers, q heads, kv heads, ffn = {args.seq_shape}; "
+                                        f"step pool of {seq.history} positions per trace before the window)"
+                                 if seq is not None else None}[args.probe],
                        "l2": f"inputs larger than L2: {eff_bytes / 2**30:.2f} GiB of per-beam KV reads per step",
                        "tree_build_s": round(t_build, 2),
                        "window": (f"steps end at the full context {wl.context} (fixed {wl.pool_bytes / 1e9:.0f} GB pool)"
@@ -597,6 +702,7 @@ def run_ours(args) -> None:
             "step_kernels_us": step_kernels_us,
             "probe_us": probe_us,
             "prune_branch_us": prune_us,
+            "scorer_fork_us": fork_us,
             "kernels": kernels,
             "capacity": capacity,
             "roofline": roofline,

@@ -262,8 +262,8 @@ gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_strea
  * events (cudaEvent_t) immediately before and after one kernel of the
  * following calls on this pool, so a caller can time that kernel alone on its
  * own stream: `which` is GB_PROF_DECODE (the split-KV decode kernel of
- * gb_decode_attention), GB_PROF_PROBE (gb_score_probe), GB_PROF_PRUNE
- * (gb_prune_branch), GB_PROF_GROUPED (the grouped shared-prefix kernel),
+ * gb_decode_attention), GB_PROF_PROBE (gb_score_probe, gb_score_mlp, or all of
+ * gb_scorer_step), GB_PROF_PRUNE (gb_prune_branch or gb_fork_slots), GB_PROF_GROUPED (the grouped shared-prefix kernel),
  * GB_PROF_PLAN (the step planner: page allocation and decode plans, layer 0),
  * GB_PROF_APPEND (the K/V append of a layer) or GB_PROF_COMBINE (the merge of
  * partial results).  Passing NULL events stops recording.  The events stay

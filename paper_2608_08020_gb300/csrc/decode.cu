@@ -102,6 +102,8 @@ __device__ __forceinline__ void unpack16x2(const uint4& u, float2* f) {
 template <int DT, int G>
 __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     k_decode(PoolView v, int layer, const void* __restrict__ qptr, float qscale, int mode, int W) {
+  pdl_wait();
+  pdl_launch_dependents();
   using T = KvTraits<DT>;
   using S = DecodeSmem<DT, G>;
   constexpr int NS = G / 2;  // scores held per lane after the reduce-scatter
@@ -428,6 +430,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 constexpr int kCombineCache = 128;
 
 __global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, float* __restrict__ out) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ float s_m[kCombineCache * 8], s_l[kCombineCache * 8];
   __shared__ float s_M[8], s_L[8];
   const int bh = blockIdx.x;
@@ -542,15 +546,15 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
   const int W = pool->decode_warps;
   const float qscale = scale * 1.4426950408889634f;  // log2(e): softmax in base 2
   prof_begin(pool, GB_PROF_DECODE, s);
-  k_decode<DT, G><<<W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s>>>(pool->view, layer, q, qscale, mode, W);
+  cudaError_t e = launch_pdl(k_decode<DT, G>, W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s, pool->view, layer, q,
+                             qscale, mode, W);
   prof_end(pool, GB_PROF_DECODE, s);
-  cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   prof_begin(pool, GB_PROF_COMBINE, s);
-  k_combine<<<pool->view.max_beams * pool->view.Hkv, 128, 0, s>>>(pool->view, mode, W, out);
+  e = launch_pdl(k_combine, pool->view.max_beams * pool->view.Hkv, 128, 0, s, pool->view, mode, W, out);
   prof_end(pool, GB_PROF_COMBINE, s);
   pool->launches += 2;
-  return cudaGetLastError();
+  return e;
 }
 
 // Split-KV decode + combine on an explicit view (plan mode 0, W warps), for callers

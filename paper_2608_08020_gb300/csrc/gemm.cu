@@ -32,6 +32,8 @@ __device__ __forceinline__ void tma_tile(uint32_t dst, const CUtensorMap* tm, in
 __global__ void __launch_bounds__(128, 1)
     k_gemm_partials(const __grid_constant__ CUtensorMap tmh, const __grid_constant__ CUtensorMap tmw, int rows, int dh,
                int H, float* __restrict__ zp, int* __restrict__ ctl) {
+  pdl_wait();
+  pdl_launch_dependents();
   extern __shared__ __align__(1024) unsigned char sm[];
   if (smem_addr(sm) & 1023) {
     if (threadIdx.x == 0) set_status(ctl, GB_ERR_UNSUPPORTED);
@@ -91,24 +93,32 @@ __global__ void __launch_bounds__(128, 1)
   }
   __syncthreads();
   ok = __syncthreads_and(tid == 0 ? ok : 1);
-  // Thread r writes row r of the partial tile (fp32), columns inside d_h only.
-  const int r = tid, row = mt * kMT + r;
-  if (ok && nkb > 0 && mbar_wait_bounded(bar + kMBarDone, 0, kWaitLimitNs)) {
-    tc_fence_after();
-    float* dst = zp + ((size_t)ks * rows + row) * dh + (size_t)nt * kNT;
+  // The partial tile goes out through shared memory (the ring is idle once the MMAs are
+  // done): thread r reads row r's 32 columns of a chunk from TMEM into a padded tile, then
+  // each warp stores whole rows, lanes over consecutive columns (rows < M, columns < N).
+  const int r = tid, lane = tid & 31;
+  float* stile = reinterpret_cast<float*>(sm);  // [128][33]
+  float* base = zp + (size_t)ks * rows * dh;
+  const bool done = ok && nkb > 0 && mbar_wait_bounded(bar + kMBarDone, 0, kWaitLimitNs);
+  const bool have = __syncthreads_and(done);  // uniform: tcgen05.ld is warp-collective
+  if (ok && nkb > 0 && !have && tid == 0) set_status(ctl, GB_ERR_TIMEOUT);
+  if (have) tc_fence_after();
 #pragma unroll 1
-    for (int c0 = 0; c0 < kNT; c0 += 32) {
+  for (int c0 = 0; c0 < kNT; c0 += 32) {
+    if (nt * kNT + c0 >= dh) break;
+    if (have) {
       float z[32];
       tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + c0, z);
-      if (row < rows) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (nt * kNT + c0 + i < dh) dst[c0 + i] = z[i];
-      }
+      for (int i = 0; i < 32; ++i) stile[r * 33 + i] = z[i];
     }
-  } else if (nkb == 0 && row < rows) {
-    float* dst = zp + ((size_t)ks * rows + row) * dh + (size_t)nt * kNT;
-    for (int c = 0; c < kNT && nt * kNT + c < dh; ++c) dst[c] = 0.f;
+    __syncthreads();
+    const int col = nt * kNT + c0 + lane;
+    for (int rr = warp; rr < kMT; rr += 4) {
+      const int row = mt * kMT + rr;
+      if (row < rows && col < dh) base[(size_t)row * dh + col] = have ? stile[rr * 33 + lane] : 0.f;
+    }
+    __syncthreads();
   }
   tc_fence_before();
   __syncthreads();
@@ -163,8 +173,7 @@ cudaError_t gemm_partials(const void* A, int M, const void* B, int N, int K, int
   CUtensorMap ta, tb;
   if (!encode_rows(&ta, A, M, K) || !encode_rows(&tb, B, N, K)) return cudaErrorInvalidValue;
   const int mtiles = (M + kMT - 1) / kMT, ntiles = (N + kNT - 1) / kNT;
-  k_gemm_partials<<<dim3(mtiles, ntiles, splits), 128, kMSmem, s>>>(ta, tb, M, N, K, P, ctl);
-  return cudaGetLastError();
+  return launch_pdl(k_gemm_partials, dim3(mtiles, ntiles, splits), 128, kMSmem, s, ta, tb, M, N, K, P, ctl);
 }
 
 }  // namespace gb

@@ -127,6 +127,8 @@ template <int G>
 __global__ void __launch_bounds__(kThreads, 1)
     k_grouped(PoolView v, const __grid_constant__ CUtensorMap tm, int layer, const __nv_bfloat16* __restrict__ q,
               float qscale, int w_oob) {
+  pdl_wait();
+  pdl_launch_dependents();
   extern __shared__ __align__(1024) unsigned char sm[];
   if (v.ctl[kCtlStepOk] == 0) return;
   const long long units = (long long)v.ctl[kCtlSegTiles] * v.Hkv;
@@ -592,11 +594,12 @@ static cudaError_t launch_grouped_t(gb_pool* pool, int layer, const void* q, flo
   const PoolView& v = pool->view;
   const float qscale = scale * 1.4426950408889634f;
   prof_begin(pool, GB_PROF_GROUPED, s);
-  k_grouped<G><<<pool->num_sms, kThreads, kSmem, s>>>(v, *reinterpret_cast<const CUtensorMap*>(pool->tmap), layer,
-                                                     static_cast<const __nv_bfloat16*>(q), qscale, pool->tmap_oob);
+  const cudaError_t e = launch_pdl(k_grouped<G>, pool->num_sms, kThreads, kSmem, s, v,
+                                   *reinterpret_cast<const CUtensorMap*>(pool->tmap), layer,
+                                   static_cast<const __nv_bfloat16*>(q), qscale, pool->tmap_oob);
   prof_end(pool, GB_PROF_GROUPED, s);
   pool->launches += 1;
-  return cudaGetLastError();
+  return e;
 }
 
 cudaError_t launch_grouped(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {

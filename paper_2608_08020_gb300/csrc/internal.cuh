@@ -5,6 +5,7 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 #include <string>
+#include <utility>
 
 #include "gambit.h"
 
@@ -127,6 +128,16 @@ __device__ __forceinline__ long long kv_elem_offset(const PoolView& v, int layer
          (long long)row * v.D;
 }
 
+// Programmatic dependent launch.  Every kernel of the library begins with pdl_wait(),
+// before any global memory access: launched normally it returns at once; launched with
+// programmatic stream serialization (launch_pdl) the kernel may be scheduled while the
+// previous kernel in the stream is still running, and pdl_wait() blocks until that
+// kernel has completed and its writes are visible - the same ordering as a plain launch,
+// without the gap between the two kernels.  pdl_launch_dependents() lets the next
+// kernel be scheduled as soon as every CTA of this one has started.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ void set_status(int* ctl, int code) {
   atomicCAS(&ctl[kCtlStatus], GB_OK, code);
 }
@@ -173,6 +184,26 @@ __device__ __forceinline__ int block_exclusive_scan(int x, int* tmp, int* total)
 }
 
 // Host side --------------------------------------------------------------------
+
+// Launch with programmatic stream serialization (see pdl_wait).  Built with -DGB_NO_PDL
+// it is a plain launch.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+#ifndef GB_NO_PDL
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+#endif
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 struct DecodeShape {
   int dtype, D, G;

@@ -26,6 +26,8 @@ __global__ void __launch_bounds__(kScoreThreads) k_mlp_score(PoolView v, const f
                                                              const float* __restrict__ w2, float b2,
                                                              const uint8_t* __restrict__ mask,
                                                              float* __restrict__ score_out) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ float red[kScoreThreads / 32];
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (!v.active[b]) {
@@ -66,7 +68,9 @@ cudaError_t launch_mlp(gb_pool* pool, const void* hidden, int H, const void* w1,
   prof_begin(pool, GB_PROF_PROBE, s);
   cudaError_t e = gemm_partials(hidden, v.max_beams, w1, dh, H, splits, v.mlp_scratch, v.ctl, s);
   if (e != cudaSuccess) return e;
-  k_mlp_score<<<v.max_beams, kScoreThreads, 0, s>>>(v, v.mlp_scratch, splits, dh, b1, w2, b2, mask, score_out);
+  e = launch_pdl(k_mlp_score, v.max_beams, kScoreThreads, 0, s, v, static_cast<const float*>(v.mlp_scratch), splits,
+                 dh, b1, w2, b2, mask, score_out);
+  if (e != cudaSuccess) return e;
   prof_end(pool, GB_PROF_PROBE, s);
   pool->launches += 2;
   return cudaGetLastError();

@@ -61,6 +61,8 @@ ScratchLayout scratch_layout(int beams, int Hkv, int W, int record_floats) {
 // Work plan for caller-owned rows (one thread per row): every row with seq_len > 0 is
 // read whole.  Also clears the status word, the one scratch value that must start at zero.
 __global__ void __launch_bounds__(1024) k_noalloc_plan(PoolView v) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ int tmp[33];
   const int b = threadIdx.x;
   const int L = b < v.max_beams ? v.seq_len[b] : 0;

@@ -134,6 +134,8 @@ __device__ void take_pages(const PoolView& v, const int* pages, int n) {
 // ---------------------------------------------------------------------------
 
 __global__ void k_init(PoolView v) {
+  pdl_wait();
+  pdl_launch_dependents();
   const long long tid = blockIdx.x * (long long)blockDim.x + threadIdx.x;
   const long long stride = (long long)gridDim.x * blockDim.x;
   for (long long w = tid; w < v.words; w += stride) {
@@ -151,6 +153,8 @@ __global__ void k_init(PoolView v) {
 
 // Reserve the prompt's pages for n root beams (one CTA).
 __global__ void __launch_bounds__(1024) k_seed_alloc(PoolView v, int n_beams, int prompt_len) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ int tmp[33];
   __shared__ int s_pages[2048];
   const int npg = (prompt_len + v.P - 1) / v.P;
@@ -182,6 +186,8 @@ __global__ void __launch_bounds__(1024) k_seed_alloc(PoolView v, int n_beams, in
 
 // Copy the prompt's K/V ([layer][T][Hkv][D]) into the pages listed in slot 0's table.
 __global__ void k_seed_write(PoolView v, int prompt_len, const char* kp, const char* vp) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int vec_per_row = v.D * v.esize / 16;
   const long long rows = (long long)v.layers * prompt_len * v.Hkv;
   const long long total = rows * vec_per_row * 2;
@@ -208,6 +214,8 @@ __global__ void k_seed_write(PoolView v, int prompt_len, const char* kp, const c
 // copy still-shared partial tail pages, advance lengths, build decode plans.
 // All or nothing: if the pool cannot supply every page the step is a no-op.
 __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, const int* seg_cover) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ int tmp[33];
   __shared__ int s_alloc[kMaxBeams];
   __shared__ int s_tail[kMaxBeams];
@@ -329,6 +337,8 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
 // Write n_tokens new K/V rows per active slot for one layer at positions
 // [seq_len - n_tokens, seq_len).  kin/vin: [n_tokens][max_beams][Hkv][D].
 __global__ void k_append(PoolView v, int layer, int n_tokens, const char* kin, const char* vin) {
+  pdl_wait();
+  pdl_launch_dependents();
   if (v.ctl[kCtlStepOk] == 0) return;
   const int vec_per_row = v.D * v.esize / 16;
   // Copy-on-write of still-shared partial tail pages, this layer's rows [0, rows).
@@ -373,6 +383,8 @@ __global__ void k_append(PoolView v, int layer, int n_tokens, const char* kin, c
 
 // Release listed slots in order (one CTA).
 __global__ void __launch_bounds__(1024) k_release(PoolView v, const int* slots, int n) {
+  pdl_wait();
+  pdl_launch_dependents();
   for (int i = 0; i < n; ++i) {
     const int s = slots[i];
     if (s < 0 || s >= v.max_beams) {
@@ -400,7 +412,9 @@ __global__ void __launch_bounds__(1024) k_release(PoolView v, const int* slots, 
   }
 }
 
-__global__ void k_clear_status(PoolView v) { v.ctl[kCtlStatus] = GB_OK; }
+__global__ void k_clear_status(PoolView v) {
+  pdl_wait();
+  pdl_launch_dependents(); v.ctl[kCtlStatus] = GB_OK; }
 
 }  // namespace gb
 
@@ -586,7 +600,8 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
   if (layer != pool->next_layer) return fail(pool, GB_ERR_STATE, "layers of a step must be called in order");
   if (layer == 0) {
     prof_begin(pool, GB_PROF_PLAN, s);
-    k_step_begin<<<1, 1024, 0, s>>>(pool->view, n_tokens, pool->view.grouped ? pool->view.seg_cover : nullptr);
+    launch_pdl(k_step_begin, 1, 1024, 0, s, pool->view, n_tokens,
+               pool->view.grouped ? pool->view.seg_cover : nullptr);
     prof_end(pool, GB_PROF_PLAN, s);
     pool->launches += 1;
     gb_status st = check_launch(pool, "step_begin");
@@ -599,8 +614,8 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
                          (pool->view.D * pool->view.esize / 16);
   const int grid = (int)std::min<long long>((vecs + 255) / 256, pool->num_sms * 8LL);
   prof_begin(pool, GB_PROF_APPEND, s);
-  k_append<<<std::max(grid, 1), 256, 0, s>>>(pool->view, layer, n_tokens, static_cast<const char*>(k),
-                                             static_cast<const char*>(v));
+  launch_pdl(k_append, std::max(grid, 1), 256, 0, s, pool->view, layer, n_tokens, static_cast<const char*>(k),
+             static_cast<const char*>(v));
   prof_end(pool, GB_PROF_APPEND, s);
   pool->launches += 1;
   gb_status st = check_launch(pool, "append");

@@ -44,6 +44,8 @@ template <int HT>
 __global__ void k_probe(PoolView v, const void* __restrict__ hidden, int H, const float* __restrict__ w,
                         float bias, const uint8_t* __restrict__ mask, float* __restrict__ score_out,
                         const float* __restrict__ scores_in) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int lane = threadIdx.x & 31;
   const int warps = blockDim.x >> 5;
   for (int b = blockIdx.x * warps + (threadIdx.x >> 5); b < v.max_beams; b += gridDim.x * warps) {
@@ -77,12 +79,14 @@ cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, in
   const int grid = (pool->view.max_beams + warps_per_block - 1) / warps_per_block;
   pool->launches += 1;
   if (scores_in == nullptr) prof_begin(pool, GB_PROF_PROBE, s);
-  if (hidden_dtype == GB_BF16)
-    k_probe<GB_BF16><<<grid, warps_per_block * 32, 0, s>>>(pool->view, hidden, H, w, bias, mask, score_out, scores_in);
-  else
-    k_probe<GB_F32><<<grid, warps_per_block * 32, 0, s>>>(pool->view, hidden, H, w, bias, mask, score_out, scores_in);
+  const cudaError_t e =
+      hidden_dtype == GB_BF16
+          ? launch_pdl(k_probe<GB_BF16>, grid, warps_per_block * 32, 0, s, pool->view, hidden, H, w, bias, mask,
+                       score_out, scores_in)
+          : launch_pdl(k_probe<GB_F32>, grid, warps_per_block * 32, 0, s, pool->view, hidden, H, w, bias, mask,
+                       score_out, scores_in);
   if (scores_in == nullptr) prof_end(pool, GB_PROF_PROBE, s);
-  return cudaGetLastError();
+  return e;
 }
 
 }  // namespace gb

@@ -28,6 +28,8 @@ __global__ void __launch_bounds__(1024) k_prune_branch(PoolView v, int C, int K,
                                                         int* __restrict__ parent_out,
                                                         uint8_t* __restrict__ pruned_out,
                                                         unsigned* __restrict__ lineage_out) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ unsigned long long keys[kMaxBeams];
   __shared__ int ord[kMaxBeams];     // rank -> slot
   __shared__ int blist[kMaxBeams];   // eligible parents in rank order
@@ -164,9 +166,12 @@ __global__ void __launch_bounds__(1024) k_prune_branch(PoolView v, int C, int K,
 // Apply a tournament decided elsewhere (another pool's parent_out): every slot s with
 // parent_of[s] >= 0 and != s becomes a child of parent_of[s] - its old references go, it
 // takes the parent's table (+1 on every page), length, mean and count, gen = 0 and a new
-// lineage id, in ascending slot order.  One CTA; the parents must not be children
-// themselves (survivors keep parent_of[p] = p).
+// lineage id, in ascending slot order.  One CTA, one warp per child (lanes over table
+// entries): reference counts change by atomics, so the end state does not depend on the
+// order; the parents must not be children themselves (survivors keep parent_of[p] = p).
 __global__ void __launch_bounds__(1024) k_fork_slots(PoolView v, const int* __restrict__ parent_of) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ int cslot[kMaxBeams], cpar[kMaxBeams];
   __shared__ int tmp[33];
   const int tid = threadIdx.x;
@@ -180,14 +185,15 @@ __global__ void __launch_bounds__(1024) k_fork_slots(PoolView v, const int* __re
     cpar[k] = p;
   }
   __syncthreads();
-  for (int c = 0; c < nchild; ++c) {
+  const int lane = tid & 31, nwarps = blockDim.x >> 5;
+  for (int c = tid >> 5; c < nchild; c += nwarps) {
     const int s = cslot[c], par = cpar[c];
     const int old_n = v.active[s] ? (v.seq_len[s] + v.P - 1) / v.P : 0;
     const int new_n = (v.seq_len[par] + v.P - 1) / v.P;
     const int m = old_n > new_n ? old_n : new_n;
     int* ts = v.tables + (size_t)s * v.max_pages;
     const int* tp = v.tables + (size_t)par * v.max_pages;
-    for (int i = tid; i < m; i += blockDim.x) {
+    for (int i = lane; i < m; i += 32) {
       const int old = i < old_n ? ts[i] : -1;
       const int nw = i < new_n ? tp[i] : -1;
       if (old == nw) continue;
@@ -215,11 +221,11 @@ cudaError_t launch_prune_branch(gb_pool* pool, int K, int fanout, int warmup, co
   const int grid = pool->view.max_beams < pool->num_sms ? pool->view.max_beams : pool->num_sms;
   prof_begin(pool, GB_PROF_PRUNE, s);
   const int C = pool->capacity > 0 ? pool->capacity : pool->view.max_beams;
-  k_prune_branch<<<grid, 1024, 0, s>>>(pool->view, C, K, fanout, warmup, elig, parent_out, pruned_out,
-                                       reinterpret_cast<unsigned*>(lineage_out));
+  const cudaError_t e = launch_pdl(k_prune_branch, grid, 1024, 0, s, pool->view, C, K, fanout, warmup, elig,
+                                   parent_out, pruned_out, reinterpret_cast<unsigned*>(lineage_out));
   prof_end(pool, GB_PROF_PRUNE, s);
   pool->launches += 1;
-  return cudaGetLastError();
+  return e;
 }
 
 }  // namespace gb
@@ -232,7 +238,9 @@ extern "C" gb_status gb_fork_slots(gb_pool* pool, const int32_t* parent_of_dev, 
   if (pool->next_layer != 0) return fail(pool, GB_ERR_STATE, "fork_slots inside an open step");
   if (pool->cfg.max_beams > kMaxBeams) return fail(pool, GB_ERR_UNSUPPORTED, "fork_slots: too many slots");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  k_fork_slots<<<1, 1024, 0, s>>>(pool->view, parent_of_dev);
+  prof_begin(pool, GB_PROF_PRUNE, s);
+  launch_pdl(k_fork_slots, 1, 1024, 0, s, pool->view, parent_of_dev);
+  prof_end(pool, GB_PROF_PRUNE, s);
   pool->launches += 1;
   gb_status st = check_launch(pool, "fork_slots");
   if (st != GB_OK) return st;

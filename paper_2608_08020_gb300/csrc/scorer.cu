@@ -166,22 +166,52 @@ __device__ __forceinline__ float sum_partials(const float* __restrict__ P, int s
 
 __device__ __forceinline__ bool row_live(const int* active, int m) { return active == nullptr || active[m] != 0; }
 
-// Input LayerNorm of Eq. 4: u[m] = LN_in(h[m]) (bf16 h, H wide).  Inactive rows give zeros.
+// Input LayerNorm of Eq. 4: u[m] = LN_in(h[m]) (bf16 h, H wide, H % 64 == 0).  Inactive
+// rows give zeros.  16-byte loads and stores (8 values); the row is staged in shared memory.
 __global__ void __launch_bounds__(kRowThreads) k_ln_in(const __nv_bfloat16* __restrict__ h, int H,
                                                        const float* __restrict__ g, const float* __restrict__ b,
                                                        const int* __restrict__ active,
                                                        __nv_bfloat16* __restrict__ u) {
+  pdl_wait();
+  pdl_launch_dependents();
   extern __shared__ float row[];
   __shared__ float red[33];
-  const int m = blockIdx.x;
-  __nv_bfloat16* out = u + (size_t)m * H;
+  const int m = blockIdx.x, nv = H / 8;
+  uint4* out = reinterpret_cast<uint4*>(u + (size_t)m * H);
   if (!row_live(active, m)) {
-    for (int i = threadIdx.x; i < H; i += blockDim.x) out[i] = __float2bfloat16_rn(0.f);
+    for (int i = threadIdx.x; i < nv; i += blockDim.x) out[i] = make_uint4(0, 0, 0, 0);
     return;
   }
-  for (int i = threadIdx.x; i < H; i += blockDim.x) row[i] = __bfloat162float(h[(size_t)m * H + i]);
-  __syncthreads();
-  layer_norm_row(row, H, g, b, out, red);
+  const uint4* in = reinterpret_cast<const uint4*>(h + (size_t)m * H);
+  float s = 0.f;
+  for (int i = threadIdx.x; i < nv; i += blockDim.x) {
+    const uint4 q = in[i];
+    const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __bfloat1622float2(p2[j]);
+      row[8 * i + 2 * j] = f.x;
+      row[8 * i + 2 * j + 1] = f.y;
+      s += f.x + f.y;
+    }
+  }
+  const float mu = block_sum(s, red) / (float)H;
+  float v = 0.f;
+  for (int i = threadIdx.x; i < H; i += blockDim.x) {
+    const float c = row[i] - mu;
+    v = fmaf(c, c, v);
+  }
+  const float r = 1.0f / sqrtf(block_sum(v, red) / (float)H + kLnEps);
+  for (int i = threadIdx.x; i < nv; i += blockDim.x) {
+    uint4 q;
+    __nv_bfloat162* p2 = reinterpret_cast<__nv_bfloat162*>(&q);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int e = 8 * i + 2 * j;
+      p2[j] = __floats2bfloat162_rn((row[e] - mu) * r * g[e] + b[e], (row[e + 1] - mu) * r * g[e + 1] + b[e + 1]);
+    }
+    out[i] = q;
+  }
 }
 
 enum RowMode { kGeluLn = 0, kResidLn = 1, kResidHead = 2 };
@@ -199,6 +229,8 @@ __global__ void __launch_bounds__(kRowThreads) k_row_epilogue(const float* __res
                                                               const float* __restrict__ w_out,
                                                               const float* __restrict__ b_out,
                                                               float* __restrict__ score) {
+  pdl_wait();
+  pdl_launch_dependents();
   extern __shared__ float row[];
   __shared__ float red[33];
   const int m = blockIdx.x;
@@ -247,6 +279,8 @@ __global__ void __launch_bounds__(kRowThreads) k_qkv_epilogue(const float* __res
                                                               __nv_bfloat16* __restrict__ q,
                                                               __nv_bfloat16* __restrict__ kn,
                                                               __nv_bfloat16* __restrict__ vn) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int m = blockIdx.x;
   const int N = (Hq + 2 * Hkv) * kHd;
   const bool live = row_live(active, m);
@@ -277,6 +311,8 @@ __global__ void __launch_bounds__(kRowThreads) k_qkv_epilogue(const float* __res
 __global__ void __launch_bounds__(kRowThreads) k_swiglu_epilogue(const float* __restrict__ P, int splits, int M, int F,
                                                                  const int* __restrict__ active,
                                                                  __nv_bfloat16* __restrict__ u) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int m = blockIdx.x;
   const bool live = row_live(active, m);
   for (int n = threadIdx.x; n < F; n += blockDim.x) {
@@ -291,6 +327,8 @@ __global__ void __launch_bounds__(kRowThreads) k_swiglu_epilogue(const float* __
 
 // Attention outputs (fp32) to the bf16 operand of W_o.
 __global__ void k_to_bf16(const float* __restrict__ a, size_t n, __nv_bfloat16* __restrict__ u) {
+  pdl_wait();
+  pdl_launch_dependents();
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
     u[i] = __float2bfloat16_rn(a[i]);
 }
@@ -299,6 +337,8 @@ __global__ void k_to_bf16(const float* __restrict__ a, size_t n, __nv_bfloat16* 
 // query head h returns the value of KV head h / G.
 __global__ void k_first_position_attention(const __nv_bfloat16* __restrict__ vn, int Hq, int G,
                                            __nv_bfloat16* __restrict__ u) {
+  pdl_wait();
+  pdl_launch_dependents();
   for (int j = threadIdx.x; j < Hq * kHd; j += blockDim.x) u[j] = vn[(j / kHd / G) * kHd + j % kHd];
 }
 
@@ -332,8 +372,8 @@ struct Run {
   template <int Mode>
   void rows(int splits, int M, const float* g, const float* b, const int* active, const float* w_out,
             const float* b_out, float* score) {
-    k_row_epilogue<Mode><<<M, kRowThreads, s.d * sizeof(float), st>>>(part(), splits, M, s.d, x(), g, b, active, u(),
-                                                                        w_out, b_out, score);
+    launch_pdl(k_row_epilogue<Mode>, M, kRowThreads, s.d * sizeof(float), st, part(), splits, M, s.d, x(), g, b,
+               active, u(), w_out, b_out, score);
     ++launches;
   }
 
@@ -353,8 +393,8 @@ struct Run {
                           (step ? 0 : (size_t)l * s.Hkv * kHd);
       // Layer 0 opens the step pool's step, which advances every length by one: the new
       // position is seq_len before layer 0 and seq_len - 1 after it.
-      k_qkv_epilogue<<<M, kRowThreads, 0, st>>>(part(), sp, M, s.Hq, s.Hkv, pos_of, l > 0 ? -1 : 0, active, q, kn,
-                                                vn);
+      launch_pdl(k_qkv_epilogue, M, kRowThreads, 0, st, part(), sp, M, s.Hq, s.Hkv, pos_of, l > 0 ? -1 : 0, active,
+                 q, kn, vn);
       ++launches;
       if (!step && l + 1 == s.L) break;  // the seed needs only each layer's k and v
       if (step) {
@@ -363,7 +403,8 @@ struct Run {
                                 reinterpret_cast<gb_stream_t>(st)) != GB_OK)
           return false;
         const size_t n = (size_t)M * s.d;
-        k_to_bf16<<<(int)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096), 256, 0, st>>>(att, n, u());
+        launch_pdl(k_to_bf16, (int)((n + 255) / 256 < 4096 ? (n + 255) / 256 : 4096), 256, 0, st,
+                   static_cast<const float*>(att), n, u());
       } else {
         k_first_position_attention<<<1, kRowThreads, 0, st>>>(vn, s.Hq, s.G, u());
       }
@@ -374,7 +415,7 @@ struct Run {
                      nullptr, nullptr);
       sp = gemm(u(), M, wt<__nv_bfloat16>(layer_tensor(l, kW13)), 2 * s.F, s.d);
       if (!sp) return false;
-      k_swiglu_epilogue<<<M, kRowThreads, 0, st>>>(part(), sp, M, s.F, active, u());
+      launch_pdl(k_swiglu_epilogue, M, kRowThreads, 0, st, part(), sp, M, s.F, active, u());
       ++launches;
       sp = gemm(u(), M, wt<__nv_bfloat16>(layer_tensor(l, kW2)), s.d, s.F);
       if (!sp) return false;
@@ -390,8 +431,8 @@ struct Run {
 
   // Eq. 4 and LN1 of layer 0 on M rows of h.
   bool input(const void* h, int M, const int* active) {
-    k_ln_in<<<M, kRowThreads, s.H * sizeof(float), st>>>(reinterpret_cast<const __nv_bfloat16*>(h), s.H, wt<float>(0),
-                                                          wt<float>(1), active, u());
+    launch_pdl(k_ln_in, M, kRowThreads, s.H * sizeof(float), st, reinterpret_cast<const __nv_bfloat16*>(h), s.H,
+               wt<float>(0), wt<float>(1), active, u());
     ++launches;
     const int sp = gemm(u(), M, wt<__nv_bfloat16>(2), s.d, s.H);
     if (!sp) return false;
@@ -469,7 +510,9 @@ extern "C" gb_status gb_scorer_step(gb_pool* step_pool, const gb_scorer_config* 
     return fail(step_pool, GB_ERR_INVALID, "scorer_step: hidden (16-byte aligned) and score_out required");
   if (!step_pool->seeded) return fail(step_pool, GB_ERR_STATE, "scorer_step: step pool not seeded");
   const int* active = step_pool->view.active;
+  prof_begin(step_pool, GB_PROF_PROBE, r.st);
   const bool ok = r.input(hidden_dev, r.s.C, active) && r.layers(r.s.C, true, active, score_out_dev);
+  if (ok) prof_end(step_pool, GB_PROF_PROBE, r.st);
   step_pool->launches += r.launches;
   st = check_launch(step_pool, "scorer_step");
   if (st != GB_OK) return st;

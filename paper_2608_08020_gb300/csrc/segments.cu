@@ -25,6 +25,8 @@ namespace gb {
 constexpr int kSegLenBuckets = 256;  // work-list entries sorted by length in 128-token tiles (longer ones share the last bucket)
 
 __global__ void k_seg_scan(PoolView v, unsigned long long gen) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int lane = threadIdx.x & 31;
   const int b = (int)((blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5);
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -81,6 +83,8 @@ done:
 }
 
 __global__ void k_seg_lead(PoolView v, unsigned long long gen) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   const int b = idx / kMaxSegDepth, k = idx % kMaxSegDepth;
   if (b >= v.max_beams || k >= v.seg_nseg[b]) return;
@@ -102,6 +106,8 @@ __global__ void k_seg_lead(PoolView v, unsigned long long gen) {
 }
 
 __global__ void k_seg_members(PoolView v) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   const int b = idx / kMaxSegDepth, k = idx % kMaxSegDepth;
   if (b >= v.max_beams || k >= v.seg_nseg[b]) return;
@@ -119,6 +125,8 @@ __global__ void k_seg_members(PoolView v) {
 // kMaxSegRecords partial records).  Entries are (segment, tile, split); every beam
 // gets the offsets of its records (one per split of each of its segments).
 __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ int tmp[33];
   __shared__ int s_split, s_total;
   __shared__ int hist[kSegLenBuckets];
@@ -222,13 +230,14 @@ cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s) {
   if (!v.grouped) return cudaSuccess;
   const unsigned long long gen = ++pool->seg_gen;
   const int warps_per_block = 8;
-  k_seg_scan<<<(v.max_beams + warps_per_block - 1) / warps_per_block, warps_per_block * 32, 0, s>>>(v, gen);
+  cudaError_t e = launch_pdl(k_seg_scan, (v.max_beams + warps_per_block - 1) / warps_per_block,
+                             warps_per_block * 32, 0, s, v, gen);
   const int n = v.max_beams * kMaxSegDepth;
-  k_seg_lead<<<(n + 255) / 256, 256, 0, s>>>(v, gen);
-  k_seg_members<<<(n + 255) / 256, 256, 0, s>>>(v);
-  k_seg_tiles<<<1, 1024, 0, s>>>(v);
+  if (e == cudaSuccess) e = launch_pdl(k_seg_lead, (n + 255) / 256, 256, 0, s, v, gen);
+  if (e == cudaSuccess) e = launch_pdl(k_seg_members, (n + 255) / 256, 256, 0, s, v);
+  if (e == cudaSuccess) e = launch_pdl(k_seg_tiles, 1, 1024, 0, s, v);
   pool->launches += 4;
-  return cudaGetLastError();
+  return e;
 }
 
 }  // namespace gb
