@@ -265,8 +265,9 @@ gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_strea
  * gb_decode_attention), GB_PROF_PROBE (gb_score_probe, gb_score_mlp, or all of
  * gb_scorer_step), GB_PROF_PRUNE (gb_prune_branch or gb_fork_slots), GB_PROF_GROUPED (the grouped shared-prefix kernel),
  * GB_PROF_PLAN (the step planner: page allocation and decode plans, layer 0),
- * GB_PROF_APPEND (the K/V append of a layer) or GB_PROF_COMBINE (the merge of
- * partial results).  Passing NULL events stops recording.  The events stay
+ * GB_PROF_APPEND (the K/V append of a layer), GB_PROF_COMBINE (the merge of
+ * partial results) or GB_PROF_ATTENTION (the attention kernels of a layer: the grouped
+ * and per-beam kernels, which run concurrently on two streams, up to the merge).  Passing NULL events stops recording.  The events stay
  * owned by the caller.  Under stream capture the records become external event
  * nodes of the graph.
  */
@@ -277,7 +278,8 @@ gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_strea
 #define GB_PROF_PLAN 4
 #define GB_PROF_APPEND 5
 #define GB_PROF_COMBINE 6
-#define GB_PROF_SLOTS 7
+#define GB_PROF_ATTENTION 7
+#define GB_PROF_SLOTS 8
 gb_status gb_pool_set_profile_events(gb_pool* pool, int which, void* start_event, void* stop_event);
 
 /*

@@ -30,7 +30,7 @@ EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_poo
            "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_score_mlp", "gb_fork_slots", "gb_scorer_sizes", "gb_scorer_seed",
            "gb_scorer_step", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
-GB_PROF_PLAN, GB_PROF_APPEND, GB_PROF_COMBINE = 4, 5, 6
+GB_PROF_PLAN, GB_PROF_APPEND, GB_PROF_COMBINE, GB_PROF_ATTENTION = 4, 5, 6, 7
 
 
 class GbPoolConfig(ctypes.Structure):

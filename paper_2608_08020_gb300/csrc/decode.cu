@@ -114,6 +114,11 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
   int* s_n = s_off + (kMaxBeams + 1);
   int* s_start = s_n + (kMaxBeams + 1);
   if (v.ctl[kCtlStepOk] == 0) return;
+  if (mode == 1) {  // beside the grouped kernel: this kernel's share of the SMs (decode_ctas)
+    const int nd = decode_ctas(v, W / kDecodeWarps);
+    if ((int)blockIdx.x >= nd) return;
+    W = nd * kDecodeWarps;
+  }
   {
     const int* off = plan_off(v, mode);
     const int* nn = plan_n(v, mode);
@@ -446,6 +451,7 @@ __global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, fl
     return;
   }
   const int Tot = plan_off(v, mode)[v.max_beams];
+  if (mode == 1) W = decode_ctas(v, W / kDecodeWarps) * kDecodeWarps;  // the warps the decode kernel used
   const int c = Tot > 0 ? (Tot + W - 1) / W : 1;
   const int off = plan_off(v, mode)[b] + h * n;
   const int first = off / c, npb = n > 0 ? (off + n - 1) / c - first + 1 : 0;  // per-beam records
@@ -535,7 +541,7 @@ __global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, fl
 
 template <int DT, int G>
 static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
-                                   cudaStream_t s) {
+                                   cudaStream_t s, cudaStream_t sd) {
   using S = DecodeSmem<DT, G>;
   static bool configured = false;
   if (!configured) {
@@ -545,11 +551,17 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
   }
   const int W = pool->decode_warps;
   const float qscale = scale * 1.4426950408889634f;  // log2(e): softmax in base 2
-  prof_begin(pool, GB_PROF_DECODE, s);
-  cudaError_t e = launch_pdl(k_decode<DT, G>, W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s, pool->view, layer, q,
+  prof_begin(pool, GB_PROF_DECODE, sd);
+  cudaError_t e = launch_pdl(k_decode<DT, G>, W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, sd, pool->view, layer, q,
                              qscale, mode, W);
-  prof_end(pool, GB_PROF_DECODE, s);
+  prof_end(pool, GB_PROF_DECODE, sd);
   if (e != cudaSuccess) return e;
+  if (sd != s) {  // join: the combine reads the per-beam kernel's records
+    e = cudaEventRecord(pool->ev_join, sd);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, pool->ev_join, 0);
+    if (e != cudaSuccess) return e;
+  }
+  prof_end(pool, GB_PROF_ATTENTION, s);
   prof_begin(pool, GB_PROF_COMBINE, s);
   e = launch_pdl(k_combine, pool->view.max_beams * pool->view.Hkv, 128, 0, s, pool->view, mode, W, out);
   prof_end(pool, GB_PROF_COMBINE, s);
@@ -596,19 +608,19 @@ cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* 
 }
 
 cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
-                          cudaStream_t s) {
+                          cudaStream_t s, cudaStream_t sd) {
   const int G = pool->view.G;
   if (pool->view.dtype == GB_BF16) {
     switch (G) {
-      case 2: return launch_decode_t<GB_BF16, 2>(pool, layer, q, scale, out, mode, s);
-      case 4: return launch_decode_t<GB_BF16, 4>(pool, layer, q, scale, out, mode, s);
-      case 8: return launch_decode_t<GB_BF16, 8>(pool, layer, q, scale, out, mode, s);
+      case 2: return launch_decode_t<GB_BF16, 2>(pool, layer, q, scale, out, mode, s, sd);
+      case 4: return launch_decode_t<GB_BF16, 4>(pool, layer, q, scale, out, mode, s, sd);
+      case 8: return launch_decode_t<GB_BF16, 8>(pool, layer, q, scale, out, mode, s, sd);
     }
   } else {
     switch (G) {
-      case 2: return launch_decode_t<GB_F32, 2>(pool, layer, q, scale, out, mode, s);
-      case 4: return launch_decode_t<GB_F32, 4>(pool, layer, q, scale, out, mode, s);
-      case 8: return launch_decode_t<GB_F32, 8>(pool, layer, q, scale, out, mode, s);
+      case 2: return launch_decode_t<GB_F32, 2>(pool, layer, q, scale, out, mode, s, sd);
+      case 4: return launch_decode_t<GB_F32, 4>(pool, layer, q, scale, out, mode, s, sd);
+      case 8: return launch_decode_t<GB_F32, 8>(pool, layer, q, scale, out, mode, s, sd);
     }
   }
   return cudaErrorInvalidValue;

@@ -133,6 +133,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (v.ctl[kCtlStepOk] == 0) return;
   const long long units = (long long)v.ctl[kCtlSegTiles] * v.Hkv;
   if (units == 0) return;
+  // When the per-beam kernel runs beside this one (decode_ctas), the CTAs past this
+  // kernel's share only take part in the end-of-launch ticket.
+  if ((int)blockIdx.x >= grouped_ctas(v, (int)gridDim.x)) {
+    if (threadIdx.x == 0 && atomicAdd(&v.ctl[kCtlGrpDone], 1) == (int)gridDim.x - 1) {
+      v.ctl[kCtlGrpNext] = 0;
+      v.ctl[kCtlGrpDone] = 0;
+      __threadfence();
+    }
+    return;
+  }
   if (smem_addr(sm) & 1023) {  // the swizzled layouts need a 1024-byte aligned base
     if (threadIdx.x == 0) set_status(v.ctl, GB_ERR_UNSUPPORTED);
     return;

@@ -121,6 +121,26 @@ __host__ __device__ inline int* plan_start(const PoolView& v, int mode) {
   return plan_off(v, mode) + 2 * (v.max_beams + 1);
 }
 
+#ifndef GB_DECODE_WEIGHT
+#define GB_DECODE_WEIGHT 120  // relative cost of a per-beam token against a grouped tile token (percent)
+#endif
+
+#ifndef GB_SPLIT_BYTES_PER_SM
+#define GB_SPLIT_BYTES_PER_SM (8ll << 20)
+#endif
+
+// A mode-1 step launches the grouped kernel and the per-beam kernel on two streams.
+// When the step's attention reads little per SM (below GB_SPLIT_BYTES_PER_SM), both
+// kernels are latency-bound and run side by side, each on its own share of the SMs: the
+// per-beam kernel takes decode_ctas(v, grid) of the `grid` CTAs (one per SM), in
+// proportion to its (16-token chunk x KV head) tokens against the grouped kernel's
+// (128-row tile x token) work per KV head, and the grouped kernel the rest.  Otherwise
+// each takes every CTA, and as each CTA needs most of an SM's shared memory the two run
+// one after the other.  Both kernels and the combine compute the same split from the
+// step's plan.
+__device__ __forceinline__ int decode_ctas(const PoolView& v, int grid);
+__device__ __forceinline__ int grouped_ctas(const PoolView& v, int grid);
+
 // Element offset of row `row` of the K (kv=0) or V (kv=1) slab of (layer, page, head).
 __device__ __forceinline__ long long kv_elem_offset(const PoolView& v, int layer, long long page,
                                                     int kv, int head, int row) {
@@ -137,6 +157,24 @@ __device__ __forceinline__ long long kv_elem_offset(const PoolView& v, int layer
 // kernel be scheduled as soon as every CTA of this one has started.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+__device__ __forceinline__ bool split_sms(const PoolView& v, long long td, long long tg) {
+  const long long bytes = (td + tg) * 2 * v.D * v.esize;
+  return td > 0 && tg > 0 && bytes < GB_SPLIT_BYTES_PER_SM * v.num_sms;
+}
+__device__ __forceinline__ int decode_ctas(const PoolView& v, int grid) {
+  const long long td = (long long)plan_off(v, 1)[v.max_beams] * kChunk;  // tokens x KV heads
+  const long long tg = (long long)v.ctl[kCtlSegTileTok] * v.Hkv;
+  if (!split_sms(v, td, tg)) return grid;
+  const long long wd = td * GB_DECODE_WEIGHT, wg = tg * 100;
+  const long long n = (wd * grid + (wd + wg) / 2) / (wd + wg);
+  return (int)(n < 1 ? 1 : (n > grid - 1 ? grid - 1 : n));
+}
+__device__ __forceinline__ int grouped_ctas(const PoolView& v, int grid) {
+  const long long td = (long long)plan_off(v, 1)[v.max_beams] * kChunk;
+  const long long tg = (long long)v.ctl[kCtlSegTileTok] * v.Hkv;
+  return split_sms(v, td, tg) ? grid - decode_ctas(v, grid) : grid;
+}
 
 __device__ __forceinline__ void set_status(int* ctl, int code) {
   atomicCAS(&ctl[kCtlStatus], GB_OK, code);
@@ -231,8 +269,15 @@ struct gb_pool {
   int tmap_oob = 0;                          // first row group past the tensor map (loads zeros)
   std::string last_error;
   unsigned long long launches = 0;          // kernels launched by this pool
+  cudaStream_t aux = nullptr;               // second stream: the per-beam kernel beside the grouped one
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   cudaEvent_t prof_start[GB_PROF_SLOTS] = {};  // caller-owned instrumentation events
   cudaEvent_t prof_stop[GB_PROF_SLOTS] = {};
+  ~gb_pool() {
+    if (ev_fork) cudaEventDestroy(ev_fork);
+    if (ev_join) cudaEventDestroy(ev_join);
+    if (aux) cudaStreamDestroy(aux);
+  }
 };
 
 namespace gb {
@@ -256,8 +301,9 @@ gb_status check_launch(gb_pool* pool, const char* what);
 
 
 // Kernel launchers implemented in the other translation units.
+// The per-beam kernel on s_decode, then (on s, after s_decode's work) the combine.
 cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
-                          cudaStream_t s);
+                          cudaStream_t s, cudaStream_t s_decode);
 cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* q, float scale, float* out,
                                cudaStream_t s);
 cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s);
