@@ -16,15 +16,20 @@
 //              over the first 32 of its S columns.  At the end of a unit the two groups
 //              exchange (m, l) through shared memory and each writes half of the merged
 //              unnormalised record (m, l, o) of its row;
-//   warp 8     producer: takes the next unit from the grid-wide counter (the work list
+//   warp 8     K producer: takes the next unit from the grid-wide counter (the work list
 //              is sorted longest first, so this is longest-processing-time-first across
 //              the CTAs), publishes it to the other roles through a 4-slot ring,
-//              gathers the unit's query rows into the Q buffer and streams K/V tiles
-//              through a 3-stage ring, one 5D TMA per page (K and V of one head),
-//              issued by several lanes at once;
+//              gathers the unit's query rows into the Q buffer and streams the K half
+//              of every tile through a 3-stage ring, one 5D TMA per page, issued by
+//              several lanes at once;
+//   warp 10    V producer: follows the same units and streams the V halves through a
+//              second 3-stage ring.  A K slot is free once S has read it, long before
+//              P.V has read the tile's V, so K runs further ahead than a joint K/V
+//              stage would let it;
 //   warp 9     MMA issuer: polls and issues S(n+1) or P.V(n), whichever is ready first;
 //              P.V takes P straight from tensor memory.
-// Handshakes are mbarriers: full/empty per stage, sched_full/sched_empty per unit slot,
+// Handshakes are mbarriers: full/empty per K stage and per V stage, sched_full/sched_empty
+// per unit slot,
 // q_full/q_empty, s_full, p_full and pv_done per double-buffered S/P tile, xch_full and
 // o_free per unit.  The last CTA to finish resets the grid-wide counters.  An S/P buffer is
 // reused by S(n+2) only after P.V(n) has been issued: the tensor core runs a CTA's MMAs
@@ -32,10 +37,12 @@
 //
 // Shared memory (dynamic only, 1024-byte aligned, 128-byte swizzle everywhere):
 //   Q     two [128 rows][64 dims] blocks (K-major A operand)                32 KiB
-//   K,V   3 stages x 16 row groups of 8 tokens: [group][K|V][half of D][8][64] 192 KiB
+//   K     3 stages x 16 row groups of 8 tokens: [group][half of D][8][64]    96 KiB
+//   V     3 stages, the same layout                                          96 KiB
 //   xch   (m, l) of both softmax groups for the unit-end merge                2 KiB
-// In a stage, K's 8-token groups sit 4096 bytes apart (Q.K^T: K-major B, SBO 4096, half
-// of D at +1024) and so do V's (P.V: MN-major B at +2048, LBO 1024, SBO 4096).
+// In a stage the 8-token groups sit 2048 bytes apart, the second half of D at +1024:
+// Q.K^T reads K as the K-major B operand (SBO 2048), P.V reads V as the MN-major B
+// operand (LBO 1024, SBO 2048).
 // Tensor memory: S/P 0 and S/P 1 (128 columns each), O_0 and O_1 (128 columns each).
 // Pages past the unit's tokens load out of bounds and are zero-filled.
 //
@@ -58,23 +65,27 @@ constexpr int kRows = 128;     // query rows per tile (MMA M)
 constexpr int kTok = 128;      // tokens per K/V tile (MMA N of Q.K^T)
 constexpr int kHalf = 64;      // tokens per softmax group (MMA K of one P.V)
 constexpr int kStages = 3;
-constexpr int kThreads = 320;
-constexpr int kProducerWarp = 8;
+constexpr int kThreads = 352;
+constexpr int kProducerWarp = 8;     // K producer, unit scheduling, Q gather
 constexpr int kMmaWarp = 9;
+constexpr int kVProducerWarp = 10;
 constexpr uint32_t kTmemCols = 512;  // S/P 0: [0, 128), S/P 1: [128, 256), O_0: [256, 384), O_1: [384, 512)
 constexpr uint32_t kTmemO = 256;
 
 constexpr int kQ = 0;                // 32 KiB
-constexpr int kKV = 32768;           // kStages x 64 KiB
-constexpr int kStage = 65536;
-constexpr int kBar = kKV + kStages * kStage;  // mbarriers and control words
-constexpr int kXch = kBar + 256;     // float [2 groups][2 (m, l)][128 rows]
+constexpr int kHalfStage = 32768;    // K (or V) of one 128-token tile of one head
+constexpr int kKRing = 32768;        // kStages x 32 KiB
+constexpr int kVRing = kKRing + kStages * kHalfStage;
+constexpr int kBar = kVRing + kStages * kHalfStage;  // mbarriers and control words
+constexpr int kXch = kBar + 512;     // float [2 groups][2 (m, l)][128 rows]
 constexpr int kSmem = kXch + 2048;
 
 // Control area (8-byte mbarriers, then words).
-constexpr int kBarFull = 0;          // [kStages]
-constexpr int kBarEmpty = kBarFull + 8 * kStages;
-constexpr int kBarQFull = kBarEmpty + 8 * kStages;
+constexpr int kBarKFull = 0;         // [kStages]
+constexpr int kBarKEmpty = kBarKFull + 8 * kStages;
+constexpr int kBarVFull = kBarKEmpty + 8 * kStages;
+constexpr int kBarVEmpty = kBarVFull + 8 * kStages;
+constexpr int kBarQFull = kBarVEmpty + 8 * kStages;
 constexpr int kBarQEmpty = kBarQFull + 8;
 constexpr int kBarSFull = kBarQEmpty + 8;            // [2]
 constexpr int kBarPFull = kBarSFull + 16;            // [2]
@@ -84,19 +95,20 @@ constexpr int kBarOFree = kBarXchFull + 8;
 constexpr int kSchedSlots = 4;
 constexpr int kBarSchedFull = kBarOFree + 8;                  // [kSchedSlots]
 constexpr int kBarSchedEmpty = kBarSchedFull + 8 * kSchedSlots;  // [kSchedSlots]
-constexpr int kSchedConsumers = 10;  // MMA S side, MMA P.V side, 8 softmax warps
+constexpr int kSchedConsumers = 11;  // MMA S side, MMA P.V side, 8 softmax warps, V producer
 constexpr int kWordSched = kBarSchedEmpty + 8 * kSchedSlots;  // int [kSchedSlots]: unit id, -1 = no more
 constexpr int kWordTmem = kWordSched + 4 * kSchedSlots;
 constexpr int kWordAbort = kWordTmem + 4;
-static_assert(kWordAbort + 4 <= 256, "control area");
+static_assert(kWordAbort + 4 <= 512, "control area");
 static_assert(kSmem <= 232448, "shared memory per block");
 
-// K and V of one page of one head by 5D TMA: coordinates {0, 0, 0, 0, w}, w = first K row / 8.
-__device__ __forceinline__ void tma_page(uint32_t dst, const CUtensorMap* tm, int w, uint32_t bar) {
+// K (kv = 0) or V (kv = 1) of one page of one head by 5D TMA: coordinates {0, 0, 0, kv, w},
+// w = first K row / 8.
+__device__ __forceinline__ void tma_page(uint32_t dst, const CUtensorMap* tm, int kv, int w, uint32_t bar) {
   asm volatile(
       "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(
           dst),
-      "l"(tm), "r"(0), "r"(0), "r"(0), "r"(0), "r"(w), "r"(bar)
+      "l"(tm), "r"(0), "r"(0), "r"(0), "r"(kv), "r"(w), "r"(bar)
       : "memory");
 }
 
@@ -153,8 +165,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + kBar + kWordAbort);
   if (tid == 0) {
     for (int i = 0; i < kStages; ++i) {
-      mbar_init(ctl + kBarFull + 8 * i, 1);
-      mbar_init(ctl + kBarEmpty + 8 * i, 1);
+      mbar_init(ctl + kBarKFull + 8 * i, 1);
+      mbar_init(ctl + kBarKEmpty + 8 * i, 1);
+      mbar_init(ctl + kBarVFull + 8 * i, 1);
+      mbar_init(ctl + kBarVEmpty + 8 * i, 1);
     }
     mbar_init(ctl + kBarQFull, 1);
     mbar_init(ctl + kBarQEmpty, 1);
@@ -185,10 +199,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int members_per_tile = kRows / G;
 
   if (warp == kProducerWarp) {
-    // ------------------------------------------------------------------ producer
+    // ------------------------------------------------------------------ K producer
     if (lane == 0) asm volatile("prefetch.tensormap [%0];" ::"l"(&tm) : "memory");
     const int ppt = kTok / v.P;                     // pages per tile (2 to 16)
-    const uint32_t page_bytes = (uint32_t)v.P * 512;  // K and V of one page of one head
+    const uint32_t page_bytes = (uint32_t)v.P * 256;  // K (or V) of one page of one head
     uint32_t n = 0;  // tiles issued
     int uidx = 0;    // units started
     bool ok = true;
@@ -239,15 +253,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (lane == 0 && n >= (uint32_t)kStages)
-          ok = wait_or_abort(ctl + kBarEmpty + 8 * st, ((n / kStages) - 1) & 1, abort_flag);
+          ok = wait_or_abort(ctl + kBarKEmpty + 8 * st, ((n / kStages) - 1) & 1, abort_flag);
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         if (!ok) break;
-        const uint32_t bar = ctl + kBarFull + 8 * st;
-        if (lane == 0) mbar_arrive_expect_tx(bar, kStage);
+        const uint32_t bar = ctl + kBarKFull + 8 * st;
+        if (lane == 0) mbar_arrive_expect_tx(bar, kHalfStage);
         __syncwarp();
         // Lane c issues page c: a TMA instruction holds its thread for a while, so the
         // lanes' copies go out in parallel.
-        if (lane < ppt) tma_page(sbase + kKV + st * kStage + lane * page_bytes, &tm, w, bar);
+        if (lane < ppt) tma_page(sbase + kKRing + st * kHalfStage + lane * page_bytes, &tm, 0, w, bar);
         if (j == 0) {
           // Query rows of the unit (after its first tile's copies are under way): row r =
           // (member, query head of this KV head); zero rows past the members.  The single
@@ -292,7 +306,56 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Drain: copies still in flight land before the CTA leaves (bounded).
     if (lane == 0 && *abort_flag) {
       for (uint32_t k = n > (uint32_t)kStages ? n - kStages : 0; k < n; ++k)
-        mbar_wait_bounded(ctl + kBarFull + 8 * (k % kStages), (k / kStages) & 1, kWaitLimitNs / 8);
+        mbar_wait_bounded(ctl + kBarKFull + 8 * (k % kStages), (k / kStages) & 1, kWaitLimitNs / 8);
+    }
+  } else if (warp == kVProducerWarp) {
+    // ------------------------------------------------------------------ V producer
+    const int ppt = kTok / v.P;
+    const uint32_t page_bytes = (uint32_t)v.P * 256;
+    uint32_t n = 0;  // tiles issued
+    bool ok = true;
+    for (int uidx = 0; ok; ++uidx) {
+      const int k = uidx & (kSchedSlots - 1);
+      if (lane == 0) ok = wait_or_abort(ctl + kBarSchedFull + 8 * k, (uidx / kSchedSlots) & 1, abort_flag);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) break;
+      const int id = sched[k];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(ctl + kBarSchedEmpty + 8 * k);
+      if (id < 0) break;
+      const Unit x = load_unit(v, id);
+      int page_l = 0;
+      for (int j = 0; j < x.ntok; ++j, ++n) {
+        const uint32_t st = n % kStages;
+        const int pb = j * ppt;
+        if ((pb & 31) == 0) {
+          const int tl = (pb + lane) * v.P;
+          page_l = tl < x.Ts ? v.tables[(size_t)x.rep * v.max_pages + x.seg_i0 + (x.tok_base + tl) / v.P] : 0;
+        }
+        int w = w_oob;
+        {
+          const int page_c = __shfl_sync(0xffffffffu, page_l, (pb + (lane & 15)) & 31);
+          const int tl = j * kTok + lane * v.P;
+          if (lane < ppt && tl < x.Ts) {
+            int page = page_c;
+            if (page < 0 || page >= v.num_pages) page = 0;  // recorded by the K producer
+            const long long slab = (((long long)layer * v.num_pages + page) * 2) * v.Hkv + x.h;
+            w = (int)(slab * v.P / 8);
+          }
+        }
+        if (lane == 0 && n >= (uint32_t)kStages)
+          ok = wait_or_abort(ctl + kBarVEmpty + 8 * st, ((n / kStages) - 1) & 1, abort_flag);
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+        if (!ok) break;
+        const uint32_t bar = ctl + kBarVFull + 8 * st;
+        if (lane == 0) mbar_arrive_expect_tx(bar, kHalfStage);
+        __syncwarp();
+        if (lane < ppt) tma_page(sbase + kVRing + st * kHalfStage + lane * page_bytes, &tm, 1, w, bar);
+      }
+    }
+    if (lane == 0 && *abort_flag) {
+      for (uint32_t k = n > (uint32_t)kStages ? n - kStages : 0; k < n; ++k)
+        mbar_wait_bounded(ctl + kBarVFull + 8 * (k % kStages), (k / kStages) & 1, kWaitLimitNs / 8);
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------------ MMA issuer
@@ -320,19 +383,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         j_s = 0;
       }
       if (j_s == 0 && !mbar_test(ctl + kBarQFull, uidx_s & 1)) return false;
-      if (!mbar_test(ctl + kBarFull + 8 * (n_s % kStages), (n_s / kStages) & 1)) return false;
+      if (!mbar_test(ctl + kBarKFull + 8 * (n_s % kStages), (n_s / kStages) & 1)) return false;
       return n_pv + 1 >= n_s;
     };
     auto issue_s = [&]() {
       const uint32_t st = n_s % kStages, sb = n_s & 1;
       tc_fence_after();
-      const uint32_t kb = sbase + kKV + st * kStage;
+      const uint32_t kb = sbase + kKRing + st * kHalfStage;
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk) {
         const uint64_t a = sdesc(sbase + kQ + (kk >> 2) * 16384 + (kk & 3) * 32, 16, 1024);
-        const uint64_t b = sdesc(kb + (kk >> 2) * 1024 + (kk & 3) * 32, 16, 4096);
+        const uint64_t b = sdesc(kb + (kk >> 2) * 1024 + (kk & 3) * 32, 16, 2048);
         mma(tmem + sb * 128, a, b, ID_S, kk > 0);
       }
+      mma_commit(ctl + kBarKEmpty + 8 * st);  // the K slot is free once S has read it
       mma_commit(ctl + kBarSFull + 8 * sb);
       if (j_s + 1 == xs.ntok) mma_commit(ctl + kBarQEmpty);  // last read of the Q buffer for this unit
       ++n_s;
@@ -369,19 +433,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         // P.V(n) needs both groups' P; a unit's first P.V also needs the previous unit's
         // accumulators read out (o_free), since it overwrites them.
         if (have_p && n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv >> 1) & 1) &&
+            mbar_test(ctl + kBarVFull + 8 * st, (n_pv / kStages) & 1) &&
             (j_p > 0 || uidx_p == 0 || mbar_test(ctl + kBarOFree, (uidx_p - 1) & 1))) {
           tc_fence_after();
-          const uint32_t vb = sbase + kKV + st * kStage + 2048;
+          const uint32_t vb = sbase + kVRing + st * kHalfStage;
 #pragma unroll
           for (int k = 0; k < 2; ++k)
 #pragma unroll
             for (int kk = 0; kk < kHalf / 16; ++kk) {
               // A = P_k (bf16 pairs, 8 columns per 16 tokens), B = V tokens [64k + 16kk, +16).
-              const uint64_t b = sdesc(vb + (k * 4 + kk) * 8192, 1024, 4096);
+              const uint64_t b = sdesc(vb + (k * 4 + kk) * 4096, 1024, 2048);
               mma_ts(tmem + kTmemO + k * 128, tmem + pb * 128 + k * 64 + kk * 8, b, ID_PV,
                      (j_p > 0 || kk > 0) ? 1u : 0u);
             }
-          mma_commit(ctl + kBarEmpty + 8 * st);
+          mma_commit(ctl + kBarVEmpty + 8 * st);
           mma_commit(ctl + kBarPvDone + 8 * pb);
           ++n_pv;
           if (++j_p == xp.ntok) {
@@ -560,10 +625,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // 5D tensor map over the whole pool, which is viewed as rows of D = 128 bf16 (256 bytes):
 // dims {64 dims, 8 rows, 2 halves of D, K|V, row groups of 8}, strides {256, 128,
-// Hkv * P * 256 (K slab to V slab), 2048} bytes, box {64, 8, 2, 2, P / 8} = K and V of
-// one page of one head.  The box lands in shared memory as [row group][K|V][half][8 rows]
-// [64 dims] with the 128-byte swizzle.  The row-group extent ends with the last K slab,
-// so every coordinate in range addresses a real K and V slab.
+// Hkv * P * 256 (K slab to V slab), 2048} bytes, box {64, 8, 2, 1, P / 8} = K (K|V
+// coordinate 0) or V (coordinate 1) of one page of one head.  The box lands in shared
+// memory as [row group][half][8 rows][64 dims] with the 128-byte swizzle.  The row-group
+// extent ends with the last K slab, so every coordinate in range addresses a real K and
+// V slab.
 bool make_kv_tensor_map(gb_pool* pool) {
   typedef CUresult (*EncodeFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -582,7 +648,7 @@ bool make_kv_tensor_map(gb_pool* pool) {
   if (rows >= (1ull << 31)) return false;
   cuuint64_t dims[5] = {64, 8, 2, 2, (rows - (unsigned long long)v.Hkv * v.P) / 8};
   cuuint64_t strides[4] = {256, 128, (cuuint64_t)v.Hkv * v.P * 256, 2048};
-  cuuint32_t box[5] = {64, 8, 2, 2, (cuuint32_t)(v.P / 8)};
+  cuuint32_t box[5] = {64, 8, 2, 1, (cuuint32_t)(v.P / 8)};
   cuuint32_t es[5] = {1, 1, 1, 1, 1};
   CUtensorMap* m = reinterpret_cast<CUtensorMap*>(pool->tmap);
   const CUresult r = encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, v.kv, dims, strides, box, es,
