@@ -3,19 +3,20 @@
 // For a segment of pages shared by g beams, the g x G query rows of one KV head
 // (G = Hq / Hkv) are stacked into one 128-row tile, so the segment's K and V are
 // read once for all of them and Q.K^T and P.V become dense contractions:
-//   S[128 x 128]  = Q[128 x 128] . K_tile^T          (tcgen05.mma kind::f16, fp32 in TMEM)
-//   O_k[128 x 128] += P_k[128 x 64] . V_tile,k        (k = 0, 1: the two 64-token halves)
+//   S[128 x 128]  = Q[128 x 128] . K_tile^T               (tcgen05.mma kind::f16, fp32 in TMEM)
+//   O[128 x 128] += P_0[128 x 64] . V_0 + P_1[128 x 64] . V_1  (the tile's two 64-token halves)
 // over 128-token tiles.  A unit of work is (segment, KV head, 128-row query tile, token
 // split); a persistent grid of one CTA per SM walks the flat unit list, and the tiles of
 // all of a CTA's units form one continuous pipeline.
 //
-// Warp roles (320 threads):
+// Warp roles (352 threads):
 //   warps 0-3  softmax group 0 and warps 4-7 softmax group 1: thread r of group k owns
-//              query row r (TMEM lane r) and tokens [64k, 64k + 64) of every tile, with
-//              its own running max m_k, sum l_k and accumulator O_k; it writes P_k (bf16)
-//              over the first 32 of its S columns.  At the end of a unit the two groups
-//              exchange (m, l) through shared memory and each writes half of the merged
-//              unnormalised record (m, l, o) of its row;
+//              query row r (TMEM lane r) and tokens [64k, 64k + 64) of every tile.  Each
+//              tile the two groups swap their row maxima through shared memory, so both
+//              keep the same running max m and their P.V products add into one
+//              accumulator O; each keeps its own sum l_k and writes P_k (bf16) over the
+//              first 32 of its S columns.  At the end of a unit the groups add their
+//              sums and each writes half of the unnormalised record (m, l, o) of its row;
 //   warp 8     K producer: takes the next unit from the grid-wide counter (the work list
 //              is sorted longest first, so this is longest-processing-time-first across
 //              the CTAs), publishes it to the other roles through a 4-slot ring,
@@ -29,21 +30,22 @@
 //   warp 9     MMA issuer: polls and issues S(n+1) or P.V(n), whichever is ready first;
 //              P.V takes P straight from tensor memory.
 // Handshakes are mbarriers: full/empty per K stage and per V stage, sched_full/sched_empty
-// per unit slot,
-// q_full/q_empty, s_full, p_full and pv_done per double-buffered S/P tile, xch_full and
-// o_free per unit.  The last CTA to finish resets the grid-wide counters.  An S/P buffer is
-// reused by S(n+2) only after P.V(n) has been issued: the tensor core runs a CTA's MMAs
-// in issue order, so P(n) has been read before S(n+2) overwrites it.
+// per unit slot, q_full/q_empty, s_full, p_full and pv_done per S/P tile (three in
+// tensor memory), max_full per tile parity, xch_full and o_free per unit.  The last CTA
+// to finish resets the grid-wide counters.  An S/P buffer is reused by S(n+3) only after
+// P.V(n) has been issued: the tensor core runs a CTA's MMAs in issue order, so P(n) has
+// been read before S(n+3) overwrites it.  With three buffers S runs two tiles ahead of
+// the softmax.
 //
 // Shared memory (dynamic only, 1024-byte aligned, 128-byte swizzle everywhere):
 //   Q     two [128 rows][64 dims] blocks (K-major A operand)                32 KiB
 //   K     3 stages x 16 row groups of 8 tokens: [group][half of D][8][64]    96 KiB
 //   V     3 stages, the same layout                                          96 KiB
-//   xch   (m, l) of both softmax groups for the unit-end merge                2 KiB
+//   xch   row maxima (and at a unit's end the sums) of both groups, per tile parity  2 KiB
 // In a stage the 8-token groups sit 2048 bytes apart, the second half of D at +1024:
 // Q.K^T reads K as the K-major B operand (SBO 2048), P.V reads V as the MN-major B
 // operand (LBO 1024, SBO 2048).
-// Tensor memory: S/P 0 and S/P 1 (128 columns each), O_0 and O_1 (128 columns each).
+// Tensor memory: S/P 0, 1, 2 (128 columns each) and O (128 columns).
 // Pages past the unit's tokens load out of bounds and are zero-filled.
 //
 // Softmax (base 2): a running max is raised only when a tile's max exceeds it by more
@@ -69,15 +71,16 @@ constexpr int kThreads = 352;
 constexpr int kProducerWarp = 8;     // K producer, unit scheduling, Q gather
 constexpr int kMmaWarp = 9;
 constexpr int kVProducerWarp = 10;
-constexpr uint32_t kTmemCols = 512;  // S/P 0: [0, 128), S/P 1: [128, 256), O_0: [256, 384), O_1: [384, 512)
-constexpr uint32_t kTmemO = 256;
+constexpr int kSBufs = 3;            // S/P tiles in tensor memory
+constexpr uint32_t kTmemCols = 512;  // S/P 0, 1, 2: [0, 384) (128 columns each), O: [384, 512)
+constexpr uint32_t kTmemO = 384;
 
 constexpr int kQ = 0;                // 32 KiB
 constexpr int kHalfStage = 32768;    // K (or V) of one 128-token tile of one head
 constexpr int kKRing = 32768;        // kStages x 32 KiB
 constexpr int kVRing = kKRing + kStages * kHalfStage;
 constexpr int kBar = kVRing + kStages * kHalfStage;  // mbarriers and control words
-constexpr int kXch = kBar + 512;     // float [2 groups][2 (m, l)][128 rows]
+constexpr int kXch = kBar + 512;     // float [2 tile parities][2 groups][128 rows]
 constexpr int kSmem = kXch + 2048;
 
 // Control area (8-byte mbarriers, then words).
@@ -87,10 +90,11 @@ constexpr int kBarVFull = kBarKEmpty + 8 * kStages;
 constexpr int kBarVEmpty = kBarVFull + 8 * kStages;
 constexpr int kBarQFull = kBarVEmpty + 8 * kStages;
 constexpr int kBarQEmpty = kBarQFull + 8;
-constexpr int kBarSFull = kBarQEmpty + 8;            // [2]
-constexpr int kBarPFull = kBarSFull + 16;            // [2]
-constexpr int kBarPvDone = kBarPFull + 16;           // [2]
-constexpr int kBarXchFull = kBarPvDone + 16;
+constexpr int kBarSFull = kBarQEmpty + 8;            // [kSBufs]
+constexpr int kBarPFull = kBarSFull + 8 * kSBufs;    // [kSBufs]
+constexpr int kBarPvDone = kBarPFull + 8 * kSBufs;   // [kSBufs]
+constexpr int kBarMaxFull = kBarPvDone + 8 * kSBufs; // [2]: the two groups' row maxima of a tile are in
+constexpr int kBarXchFull = kBarMaxFull + 16;
 constexpr int kBarOFree = kBarXchFull + 8;
 constexpr int kSchedSlots = 4;
 constexpr int kBarSchedFull = kBarOFree + 8;                  // [kSchedSlots]
@@ -172,11 +176,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(ctl + kBarQFull, 1);
     mbar_init(ctl + kBarQEmpty, 1);
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kSBufs; ++i) {
       mbar_init(ctl + kBarSFull + 8 * i, 1);
       mbar_init(ctl + kBarPFull + 8 * i, 8);
       mbar_init(ctl + kBarPvDone + 8 * i, 1);
     }
+    for (int i = 0; i < 2; ++i) mbar_init(ctl + kBarMaxFull + 8 * i, 8);
     mbar_init(ctl + kBarXchFull, 8);
     mbar_init(ctl + kBarOFree, 8);
     for (int i = 0; i < kSchedSlots; ++i) {
@@ -206,18 +211,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t n = 0;  // tiles issued
     int uidx = 0;    // units started
     bool ok = true;
-    auto fetch = [&]() -> long long {
-      long long id = 0;
-      if (lane == 0) id = atomicAdd(&v.ctl[kCtlGrpNext], 1);
-      return __shfl_sync(0xffffffffu, id, 0);
-    };
+    // Units come from the grid-wide counter one unit ahead: the request for the next unit
+    // goes out when this one starts, so its latency hides behind this unit's tiles.  A
+    // unit (or the end, -1) is published in slot uidx % kSchedSlots once every role has
+    // read the unit that slot held before.
+    int pending = 0;
+    if (lane == 0) pending = atomicAdd(&v.ctl[kCtlGrpNext], 1);
     for (;; ++uidx) {
       if (!ok || *abort_flag) break;
-      // The next unit is taken only once this CTA has issued every copy of the previous
-      // one (the producer runs a few tiles ahead of the tensor core), so a unit goes to
-      // the CTA that is about to be free.  It (or the end, -1) is published in slot
-      // uidx % kSchedSlots once every role has read the unit that slot held before.
-      const long long u = fetch();
+      const long long u = __shfl_sync(0xffffffffu, pending, 0);
+      if (lane == 0 && u < units) pending = atomicAdd(&v.ctl[kCtlGrpNext], 1);
       const int k = uidx & (kSchedSlots - 1);
       if (lane == 0 && uidx >= kSchedSlots)
         ok = wait_or_abort(ctl + kBarSchedEmpty + 8 * k, ((uidx / kSchedSlots) - 1) & 1, abort_flag);
@@ -272,9 +275,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             ++n;
             break;
           }
-          // Lane l takes rows l, l + 32, l + 64, l + 96: their member beams first, then the
-          // rows two at a time (32 loads of 16 bytes in flight per lane).
-          const uint4* qrow[kRows / 32];
+          // Lane l takes rows l, l + 32, l + 64, l + 96: their member beams first, then all
+          // 64 16-byte pieces of its rows as asynchronous copies into the swizzled layout,
+          // so the whole 32 KiB is in flight at once; rows past the members are zeroed.
+          const char* qrow[kRows / 32];
           bool qvalid[kRows / 32];
 #pragma unroll
           for (int i = 0; i < kRows / 32; ++i) {
@@ -282,21 +286,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int m = x.t * members_per_tile + r / G, gg = r % G;
             qvalid[i] = m < x.g;
             const int b = qvalid[i] ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
-            qrow[i] = reinterpret_cast<const uint4*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
+            qrow[i] = reinterpret_cast<const char*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
           }
 #pragma unroll
-          for (int i0 = 0; i0 < kRows / 32; i0 += 2) {
-            uint4 buf[2][16];
+          for (int i = 0; i < kRows / 32; ++i)
 #pragma unroll
-            for (int ii = 0; ii < 2; ++ii)
-#pragma unroll
-              for (int c = 0; c < 16; ++c) buf[ii][c] = qvalid[i0 + ii] ? qrow[i0 + ii][c] : make_uint4(0, 0, 0, 0);
-#pragma unroll
-            for (int ii = 0; ii < 2; ++ii)
-#pragma unroll
-              for (int c = 0; c < 16; ++c)
-                *reinterpret_cast<uint4*>(sm + kQ + (c >> 3) * 16384 + swz(lane + 32 * (i0 + ii), (c & 7) * 8)) = buf[ii][c];
-          }
+            for (int c = 0; c < 16; ++c) {
+              const uint32_t dst = sbase + kQ + (c >> 3) * 16384 + swz(lane + 32 * i, (c & 7) * 8);
+              if (qvalid[i])
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(qrow[i] + 16 * c) : "memory");
+              else
+                *reinterpret_cast<uint4*>(sm + (dst - sbase)) = make_uint4(0, 0, 0, 0);
+            }
+          asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) mbar_arrive(ctl + kBarQFull);
@@ -384,10 +386,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (j_s == 0 && !mbar_test(ctl + kBarQFull, uidx_s & 1)) return false;
       if (!mbar_test(ctl + kBarKFull + 8 * (n_s % kStages), (n_s / kStages) & 1)) return false;
-      return n_pv + 1 >= n_s;
+      return n_pv + (kSBufs - 1) >= n_s;
     };
     auto issue_s = [&]() {
-      const uint32_t st = n_s % kStages, sb = n_s & 1;
+      const uint32_t st = n_s % kStages, sb = n_s % kSBufs;
       tc_fence_after();
       const uint32_t kb = sbase + kKRing + st * kHalfStage;
 #pragma unroll
@@ -429,10 +431,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             progressed = true;
           }
         }
-        const uint32_t pb = n_pv & 1, st = n_pv % kStages;
+        const uint32_t pb = n_pv % kSBufs, st = n_pv % kStages;
         // P.V(n) needs both groups' P; a unit's first P.V also needs the previous unit's
-        // accumulators read out (o_free), since it overwrites them.
-        if (have_p && n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv >> 1) & 1) &&
+        // accumulator read out (o_free), since it overwrites it.
+        if (have_p && n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv / kSBufs) & 1) &&
             mbar_test(ctl + kBarVFull + 8 * st, (n_pv / kStages) & 1) &&
             (j_p > 0 || uidx_p == 0 || mbar_test(ctl + kBarOFree, (uidx_p - 1) & 1))) {
           tc_fence_after();
@@ -443,8 +445,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int kk = 0; kk < kHalf / 16; ++kk) {
               // A = P_k (bf16 pairs, 8 columns per 16 tokens), B = V tokens [64k + 16kk, +16).
               const uint64_t b = sdesc(vb + (k * 4 + kk) * 4096, 1024, 2048);
-              mma_ts(tmem + kTmemO + k * 128, tmem + pb * 128 + k * 64 + kk * 8, b, ID_PV,
-                     (j_p > 0 || kk > 0) ? 1u : 0u);
+              mma_ts(tmem + kTmemO, tmem + pb * 128 + k * 64 + kk * 8, b, ID_PV,
+                     (j_p > 0 || k > 0 || kk > 0) ? 1u : 0u);
             }
           mma_commit(ctl + kBarVEmpty + 8 * st);
           mma_commit(ctl + kBarPvDone + 8 * pb);
@@ -469,18 +471,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!alive) {
         // Let issued MMAs finish before the tensor memory is freed (bounded).
-        if (n_pv > 0) mbar_wait_bounded(ctl + kBarPvDone + 8 * ((n_pv - 1) & 1), ((n_pv - 1) >> 1) & 1, kWaitLimitNs / 8);
-        if (n_s > 0) mbar_wait_bounded(ctl + kBarSFull + 8 * ((n_s - 1) & 1), ((n_s - 1) >> 1) & 1, kWaitLimitNs / 8);
+        if (n_pv > 0)
+          mbar_wait_bounded(ctl + kBarPvDone + 8 * ((n_pv - 1) % kSBufs), ((n_pv - 1) / kSBufs) & 1, kWaitLimitNs / 8);
+        if (n_s > 0)
+          mbar_wait_bounded(ctl + kBarSFull + 8 * ((n_s - 1) % kSBufs), ((n_s - 1) / kSBufs) & 1, kWaitLimitNs / 8);
       }
     }
     __syncwarp();
   } else {
     // ------------------------------------------------------------------ softmax (warps 0-7)
+    // Both groups keep the same running max per row (they swap their tile maxima through
+    // shared memory), so their P.V products add into one accumulator O.
     const int grp = warp >> 2;           // softmax group: tokens [64 grp, 64 grp + 64) of each tile
     const int r = tid & 127;             // query row / TMEM lane
     const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
-    const uint32_t o_own = tmem + kTmemO + grp * 128 + lane_base;
-    float* xch = reinterpret_cast<float*>(sm + kXch);
+    const uint32_t o_half = tmem + kTmemO + grp * 64 + lane_base;  // this group's half of O's columns
+    float* xch = reinterpret_cast<float*>(sm + kXch);  // [tile parity][group][row]
     uint32_t n = 0;
     int uidx = 0;
     bool alive = true;
@@ -494,17 +500,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Unit x = load_unit(v, id);
       float m_ref = -INFINITY, l = 0.f;
       for (int j = 0; j < x.ntok; ++j, ++n) {
-        const uint32_t sb = n & 1;
+        const uint32_t sb = n % kSBufs;
         const uint32_t sp_addr = tmem + sb * 128 + grp * 64 + lane_base;
-        if (!wait_or_abort(ctl + kBarSFull + 8 * sb, (n >> 1) & 1, abort_flag)) { alive = false; break; }
+        if (!wait_or_abort(ctl + kBarSFull + 8 * sb, (n / kSBufs) & 1, abort_flag)) { alive = false; break; }
         tc_fence_after();
         const int valid = min(max(x.Ts - j * kTok - grp * kHalf, 0), kHalf);  // this group's tokens in the tile
-        uint32_t pw[kHalf / 2];
-        if (valid == 0) {
-#pragma unroll
-          for (int i = 0; i < kHalf / 2; ++i) pw[i] = 0u;
-        } else {
-          float sv[kHalf];
+        float sv[kHalf];
+        float mt_own = -INFINITY;
+        if (valid > 0) {
           tmem_ld32(sp_addr, sv);
           tmem_ld32(sp_addr + 32, sv + 32);
           if (valid < kHalf) {  // only a unit's last tile reaches past its tokens
@@ -513,46 +516,69 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (c >= valid) sv[c] = -INFINITY;
           }
           // Max on the raw scores; qscale > 0, so it scales to the max in log2 units.
-          float mr0 = sv[0], mr1 = sv[1];
+          float mr0 = sv[0], mr1 = sv[1], mr2 = sv[2], mr3 = sv[3];
 #pragma unroll
-          for (int c = 2; c < kHalf; c += 2) {
+          for (int c = 4; c < kHalf; c += 4) {
             mr0 = fmaxf(mr0, sv[c]);
             mr1 = fmaxf(mr1, sv[c + 1]);
+            mr2 = fmaxf(mr2, sv[c + 2]);
+            mr3 = fmaxf(mr3, sv[c + 3]);
           }
-          const float mt = fmaxf(mr0, mr1) * qscale;
-          const bool raise = mt > m_ref + 8.f;
-          if (j > 0 && __any_sync(0xffffffffu, raise)) {
-            // O_k must hold P.V(n-1) and nothing newer before it is rescaled.
-            if (!wait_or_abort(ctl + kBarPvDone + 8 * ((n - 1) & 1), ((n - 1) >> 1) & 1, abort_flag)) {
-              alive = false;
-              break;
-            }
-            tc_fence_after();
-            const float alpha = raise ? exp2f(m_ref - mt) : 1.f;
+          mt_own = fmaxf(fmaxf(mr0, mr1), fmaxf(mr2, mr3)) * qscale;
+        }
+        // The tile's row max over both groups: slot n & 1 is rewritten two tiles later,
+        // after every warp has passed this tile's barrier, so after it has been read.
+        const int slot = n & 1;
+        xch[(slot * 2 + grp) * 128 + r] = mt_own;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(ctl + kBarMaxFull + 8 * slot);
+        if (!wait_or_abort(ctl + kBarMaxFull + 8 * slot, (n >> 1) & 1, abort_flag)) { alive = false; break; }
+        const float mt = fmaxf(mt_own, xch[(slot * 2 + 1 - grp) * 128 + r]);
+        const bool raise = mt > m_ref + 8.f;
+        if (j > 0 && __any_sync(0xffffffffu, raise)) {
+          // O must hold P.V(n-1) and nothing newer before it is rescaled; each group
+          // rescales its half of the columns.
+          if (!wait_or_abort(ctl + kBarPvDone + 8 * ((n - 1) % kSBufs), ((n - 1) / kSBufs) & 1, abort_flag)) {
+            alive = false;
+            break;
+          }
+          tc_fence_after();
+          const float alpha = raise ? exp2f(m_ref - mt) : 1.f;
 #pragma unroll 1
-            for (int c0 = 0; c0 < 128; c0 += 32) {
-              float o[32];
-              tmem_ld32(o_own + c0, o);
+          for (int c0 = 0; c0 < 64; c0 += 32) {
+            float o[32];
+            tmem_ld32(o_half + c0, o);
 #pragma unroll
-              for (int i = 0; i < 32; ++i) o[i] *= alpha;
-              tmem_st32(o_own + c0, o);
-            }
-            if (raise) l *= alpha;
+            for (int i = 0; i < 32; ++i) o[i] *= alpha;
+            tmem_st32(o_half + c0, o);
           }
-          if (raise) m_ref = mt;
-          const float neg_m = -m_ref;
-          float l0 = 0.f, l1 = 0.f;
+          if (raise) l *= alpha;
+        }
+        if (raise) m_ref = mt;
+        uint32_t pw[kHalf / 2];
+        if (valid == 0) {
 #pragma unroll
-          for (int c = 0; c < kHalf; c += 2) {
+          for (int i = 0; i < kHalf / 2; ++i) pw[i] = 0u;
+        } else {
+          const float neg_m = -m_ref;
+          float l0 = 0.f, l1 = 0.f, l2 = 0.f, l3 = 0.f;
+#pragma unroll
+          for (int c = 0; c < kHalf; c += 4) {
             // p = 2^(s * qscale - m); masked scores give 2^-inf = 0.
             const float p0 = ex2_approx(fmaf(sv[c], qscale, neg_m));
             const float p1 = ex2_approx(fmaf(sv[c + 1], qscale, neg_m));
-            const __nv_bfloat162 pr = __floats2bfloat162_rn(p0, p1);
-            pw[c / 2] = *reinterpret_cast<const uint32_t*>(&pr);
+            const float p2 = ex2_approx(fmaf(sv[c + 2], qscale, neg_m));
+            const float p3 = ex2_approx(fmaf(sv[c + 3], qscale, neg_m));
+            const __nv_bfloat162 pr0 = __floats2bfloat162_rn(p0, p1);
+            const __nv_bfloat162 pr1 = __floats2bfloat162_rn(p2, p3);
+            pw[c / 2] = *reinterpret_cast<const uint32_t*>(&pr0);
+            pw[c / 2 + 1] = *reinterpret_cast<const uint32_t*>(&pr1);
             l0 += p0;
             l1 += p1;
+            l2 += p2;
+            l3 += p3;
           }
-          l += l0 + l1;
+          l += (l0 + l1) + (l2 + l3);
         }
         tmem_st32u(sp_addr, pw);  // P_k over the first 32 of this group's S columns
         tc_fence_before();
@@ -560,48 +586,44 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(ctl + kBarPFull + 8 * sb);
       }
       if (!alive) break;
-      // Unit end: both accumulators are final once P.V of the last tile has completed.
+      // Unit end: O is final once P.V of the last tile has completed.  The groups add their
+      // row sums (same max); slot n & 1 is free (its last reader passed the previous tile).
       const uint32_t last = n - 1;
-      if (!wait_or_abort(ctl + kBarPvDone + 8 * (last & 1), (last >> 1) & 1, abort_flag)) break;
+      if (!wait_or_abort(ctl + kBarPvDone + 8 * (last % kSBufs), (last / kSBufs) & 1, abort_flag)) break;
       tc_fence_after();
-      xch[(grp * 2 + 0) * 128 + r] = m_ref;
-      xch[(grp * 2 + 1) * 128 + r] = l;
+      const int slot = n & 1;
+      xch[(slot * 2 + grp) * 128 + r] = l;
       __syncwarp();
       if (lane == 0) mbar_arrive(ctl + kBarXchFull);
       if (!wait_or_abort(ctl + kBarXchFull, uidx & 1, abort_flag)) break;
-      const float m_o = xch[((1 - grp) * 2 + 0) * 128 + r], l_o = xch[((1 - grp) * 2 + 1) * 128 + r];
-      const float m0 = grp == 0 ? m_ref : m_o, l0 = grp == 0 ? l : l_o;
-      const float m1 = grp == 0 ? m_o : m_ref, l1 = grp == 0 ? l_o : l;
-      const float mm = fmaxf(m0, m1);
-      const float a0 = m0 == -INFINITY ? 0.f : exp2f(m0 - mm);
-      const float a1 = m1 == -INFINITY ? 0.f : exp2f(m1 - mm);
+      const float l_all = l + xch[(slot * 2 + 1 - grp) * 128 + r];
       const int m = x.t * members_per_tile + r / G, gg = r % G;
       const int bk = m < x.g ? v.seg_members[x.moff + m] : 0;
       const int b = bk / kMaxSegDepth;
       const int r_idx = v.seg_rec_off[bk] + x.sp;
       const bool has = m < x.g && r_idx < kMaxSegRecords;
       float* rec = v.grec + (((size_t)b * kMaxSegRecords + r_idx) * v.Hkv + x.h) * v.record_floats;
-      // Group k writes columns [64k, 64k + 64) of the merged output.
+      // Group k writes columns [64k, 64k + 64) of the output.
 #pragma unroll 1
-      for (int c0 = grp * 64; c0 < grp * 64 + 64; c0 += 32) {  // warp-collective loads: every lane takes part
-        float o0[32], o1[32];
-        tmem_ld32(tmem + kTmemO + c0 + lane_base, o0);
-        tmem_ld32(tmem + kTmemO + 128 + c0 + lane_base, o1);
+      for (int c0 = 0; c0 < 64; c0 += 32) {  // warp-collective loads: every lane takes part
+        float o[32];
+        tmem_ld32(o_half + c0, o);
         if (has) {
 #pragma unroll
           for (int i = 0; i < 32; i += 4)
-            *reinterpret_cast<float4*>(rec + gg * 128 + c0 + i) =
-                make_float4(o0[i] * a0 + o1[i] * a1, o0[i + 1] * a0 + o1[i + 1] * a1, o0[i + 2] * a0 + o1[i + 2] * a1,
-                            o0[i + 3] * a0 + o1[i + 3] * a1);
+            *reinterpret_cast<float4*>(rec + gg * 128 + grp * 64 + c0 + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
         }
       }
       if (has && grp == 0) {
-        rec[G * 128 + gg] = mm;
-        rec[G * 128 + G + gg] = l0 * a0 + l1 * a1;
+        rec[G * 128 + gg] = m_ref;
+        rec[G * 128 + G + gg] = l_all;
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(ctl + kBarOFree);
+      // Every warp has read this unit's sums before the next unit's first tile rewrites
+      // the exchange slot.
+      if (!wait_or_abort(ctl + kBarOFree, uidx & 1, abort_flag)) break;
     }
   }
 
