@@ -288,13 +288,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int b = qvalid[i] ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
             qrow[i] = reinterpret_cast<const char*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
           }
+          // Query rows are read by every unit of their beams: keep them in L2 against the
+          // stream of K/V tiles (evict-last).
+          const uint64_t qpol = policy_evict_last();
 #pragma unroll
           for (int i = 0; i < kRows / 32; ++i)
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
               const uint32_t dst = sbase + kQ + (c >> 3) * 16384 + swz(lane + 32 * i, (c & 7) * 8);
               if (qvalid[i])
-                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(qrow[i] + 16 * c) : "memory");
+                asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2;" ::"r"(dst),
+                             "l"(qrow[i] + 16 * c), "l"(qpol)
+                             : "memory");
               else
                 *reinterpret_cast<uint4*>(sm + (dst - sbase)) = make_uint4(0, 0, 0, 0);
             }
