@@ -169,10 +169,18 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     it.i = r % it.n;
   }
   const uint64_t pol = policy_evict_first();
+  // Page ids come from the block table 32 chunks at a time (lane l loads the page of chunk
+  // i0 + l of the beam, one coalesced load) and are handed out by shuffles, so a chunk's
+  // refill does not wait on a table load of its own.  Called by the whole warp.
+  int pw_b = -1, pw_i0 = 0, pw_lane = 0;
   auto load_page = [&](const ChunkIter& q) -> int {
-    const int tok = q.tok0 + q.i * kChunk;
-    int page = v.tables[(size_t)q.b * v.max_pages + tok / v.P];
-    return page;
+    if (q.b != pw_b || q.i < pw_i0 || q.i >= pw_i0 + 32) {
+      pw_b = q.b;
+      pw_i0 = q.i;
+      const int i = pw_i0 + lane;
+      pw_lane = i < q.n ? v.tables[(size_t)q.b * v.max_pages + (q.tok0 + i * kChunk) / v.P] : 0;
+    }
+    return __shfl_sync(0xffffffffu, pw_lane, q.i - pw_i0);
   };
   auto issue = [&](const ChunkIter& q, int page, int stage) {
     if (lane == 0) {
