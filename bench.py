@@ -309,6 +309,13 @@ def capacity_search(wl, dev) -> dict:
     return {"pool_pages": pages, "pool_bytes": wl.pool_bytes, "copied_beams": copied,
             "forked_beams_configured": wl.beams, "forked_beams_configured_fit": lo >= wl.beams,
             "forked_beams_max_seed0": lo}
+def bracketed_steps(W: int, K: int, event_stride: int, breakdown: bool):
+    """(stride, steps) of the timed steps whose kernels the library brackets with events:
+    every step under --breakdown, else every event_stride-th (0: about 32 of the K)."""
+    stride = 1 if breakdown else max(1, event_stride if event_stride > 0 else K // 32)
+    return stride, [i for i in range(W, W + K) if (i - W) % stride == 0]
+
+
 def build_seq_scorer(args, wl, g, dev, n_rounds_after: int):
     """The sequence scorer with seeded random weights and its step pool, seeded with the
     prompt's final hidden state and stepped once per tournament round already in the tree
@@ -457,8 +464,7 @@ def run_ours(args) -> None:
         b.record(stream)
         return a, b
     timed_rounds = [i for i in range(W, W + K) if is_round(i)]
-    stride = 1 if args.breakdown else max(1, args.event_stride if args.event_stride > 0 else K // 32)
-    inst = [i for i in range(W, W + K) if (i - W) % stride == 0]   # steps whose kernels are bracketed
+    stride, inst = bracketed_steps(W, K, args.event_stride, args.breakdown)
     profs = {i: {} for i in range(W, W + K)}
     for i in inst:
         profs[i].update({"dec": [ev_pair() for _ in range(NL)], "gr": [ev_pair() for _ in range(NL)],

@@ -22,7 +22,7 @@ def _lib():
     return binding, binding.load()
 
 
-def test_header_declares_the_north_star_calls():
+def test_header_declares_the_hot_path_calls():
     names = declared_functions()
     for n in ("gb_pool_init", "gb_decode_attention", "gb_score_probe", "gb_prune_branch", "gb_release"):
         assert n in names
