@@ -309,6 +309,60 @@ def capacity_search(wl, dev) -> dict:
     return {"pool_pages": pages, "pool_bytes": wl.pool_bytes, "copied_beams": copied,
             "forked_beams_configured": wl.beams, "forked_beams_configured_fit": lo >= wl.beams,
             "forked_beams_max_seed0": lo}
+class _Cudart:
+    """The CUDA runtime calls the end-to-end leg issues per step (copies between pinned host
+    memory and the device, events between the compute and copy streams), called directly:
+    from Python they cost a fraction of the equivalent torch calls."""
+    H2D, D2H = 1, 2
+
+    def __init__(self):
+        import ctypes
+        import ctypes.util
+        lib = None
+        for name in ("libcudart.so.13", "libcudart.so.12", ctypes.util.find_library("cudart") or "libcudart.so"):
+            try:
+                lib = ctypes.CDLL(name)
+                break
+            except OSError:
+                continue
+        if lib is None:
+            raise RuntimeError("the CUDA runtime library is not loadable")
+        P, Z, I, U = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_uint
+        self._ct = ctypes
+        self._copy = lib.cudaMemcpyAsync
+        self._copy.argtypes = [P, P, Z, I, P]
+        self._rec = lib.cudaEventRecord
+        self._rec.argtypes = [P, P]
+        self._wait = lib.cudaStreamWaitEvent
+        self._wait.argtypes = [P, P, U]
+        self._create = lib.cudaEventCreateWithFlags
+        self._create.argtypes = [P, U]
+        self._destroy = lib.cudaEventDestroy
+        self._destroy.argtypes = [P]
+
+    @staticmethod
+    def _ok(code, what):
+        if code != 0:
+            raise RuntimeError(f"{what} failed with CUDA error {code}")
+
+    def event(self):
+        e = self._ct.c_void_p()
+        self._ok(self._create(self._ct.byref(e), 2), "cudaEventCreateWithFlags")  # cudaEventDisableTiming
+        return e.value
+
+    def destroy(self, e):
+        self._destroy(e)
+
+    def copy(self, dst, src, n, kind, stream):
+        self._ok(self._copy(dst, src, n, kind, stream), "cudaMemcpyAsync")
+
+    def record(self, e, stream):
+        self._ok(self._rec(e, stream), "cudaEventRecord")
+
+    def wait(self, stream, e):
+        self._ok(self._wait(stream, e, 0), "cudaStreamWaitEvent")
+
+
 def bracketed_steps(W: int, K: int, event_stride: int, breakdown: bool):
     """(stride, steps) of the timed steps whose kernels the library brackets with events:
     every step under --breakdown, else every event_stride-th (0: about 32 of the K)."""
@@ -631,8 +685,14 @@ def run_ours(args) -> None:
         r_h = {n: [torch.empty(C, dtype=t.dtype).pin_memory() for t in (g.scores, g.parent, g.pruned, g.lineage)]
                for n, i in enumerate(sl) if is_round(i)}
         cs = torch.cuda.Stream(device=dev)
-        ev = lambda: torch.cuda.Event()
-        loaded, done, outfree = ([ev() for _ in range(2)] for _ in range(3))
+        rt = _Cudart()
+        S, CS = stream.cuda_stream, cs.cuda_stream
+        loaded, done, outfree = ([rt.event() for _ in range(2)] for _ in range(3))
+        ev_fork, ev_join = rt.event(), rt.event()
+        out_bytes = dout[0].numel() * dout[0].element_size()
+        # Pointers of every buffer, layer and tensor, so a decode-only step is plain C calls.
+        ptrs = [[(views[b][0][l].data_ptr(), views[b][1][l].data_ptr(), views[b][2][l].data_ptr(),
+                  dout[b][l].data_ptr()) for l in range(NL)] for b in range(2)]
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
@@ -642,48 +702,58 @@ def run_ours(args) -> None:
         def load(n):                         # inputs of e2e step n into buffer n % 2 (copy stream)
             nonlocal h2d
             b = n % 2
-            with torch.cuda.stream(cs):
-                if n >= 2:
-                    cs.wait_event(done[b])
-                din[b].copy_(hin[n], non_blocking=True)
-                h2d += in_bytes
-                if is_round(sl[n]):
-                    h_d[b].copy_(hh[h_index[sl[n]]], non_blocking=True)
-                    h2d += hh[0].numel() * hh.element_size()
-                loaded[b].record(cs)
+            if n >= 2:
+                rt.wait(CS, done[b])
+            rt.copy(din[b].data_ptr(), hin[n].data_ptr(), in_bytes, rt.H2D, CS)
+            h2d += in_bytes
+            if is_round(sl[n]):
+                nb = hh[0].numel() * hh.element_size()
+                rt.copy(h_d[b].data_ptr(), hh[h_index[sl[n]]].data_ptr(), nb, rt.H2D, CS)
+                h2d += nb
+            rt.record(loaded[b], CS)
 
         e0.record(stream)
         t_host = time.perf_counter()
-        cs.wait_stream(stream)
+        rt.record(ev_fork, S)
+        rt.wait(CS, ev_fork)
         load(0)
         for n, i in enumerate(sl):
             b = n % 2
             if n + 1 < K:
                 load(n + 1)
-            stream.wait_event(loaded[b])
+            rt.wait(S, loaded[b])
             if n >= 2:
-                stream.wait_event(outfree[b])
-            step(i, *views[b], h_d[b], o=dout[b])
-            done[b].record(stream)
-            with torch.cuda.stream(cs):
-                cs.wait_event(done[b])
-                o_h[b].copy_(dout[b], non_blocking=True)
-                d2h += o_h[b].numel() * o_h[b].element_size()
-                if is_round(i):
-                    for host, dev_t in zip(r_h[n], (g.scores, g.parent, g.pruned, g.lineage)):
-                        host.copy_(dev_t, non_blocking=True)
-                        d2h += host.numel() * host.element_size()
-                outfree[b].record(cs)
-        stream.wait_stream(cs)
+                rt.wait(S, outfree[b])
+            if is_round(i):
+                step(i, *views[b], h_d[b], o=dout[b])
+            else:
+                for l in range(NL):
+                    qp, kp, vp, op = ptrs[b][l]
+                    B.gb_decode_attention(pool.handle, l, qp, kp, vp, wl.attn_scale, op, flags, S)
+            rt.record(done[b], S)
+            rt.wait(CS, done[b])
+            rt.copy(o_h[b].data_ptr(), dout[b].data_ptr(), out_bytes, rt.D2H, CS)
+            d2h += out_bytes
+            if is_round(i):
+                for host, dev_t in zip(r_h[n], (g.scores, g.parent, g.pruned, g.lineage)):
+                    nb = host.numel() * host.element_size()
+                    rt.copy(host.data_ptr(), dev_t.data_ptr(), nb, rt.D2H, CS)
+                    d2h += nb
+            rt.record(outfree[b], CS)
+        rt.record(ev_join, CS)
+        rt.wait(S, ev_join)
         e1.record(stream)
         t_host = time.perf_counter() - t_host
         torch.cuda.synchronize()
+        for e in loaded + done + outfree + [ev_fork, ev_join]:
+            rt.destroy(e)
         e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
         e2e = {"value": job_value(world, C, K, e_ms), "unit": "beam-tokens/s", "h2d_bytes_per_step": int(h2d // K),
                "d2h_bytes_per_step": int(d2h // K), "ms_per_step": e_ms / K,
                "host_issue_us_per_step": t_host / K * 1e6,
-               "path": "eager calls of the pool API; inputs copied from pinned host memory and outputs read back "
-                       "every step, on a copy stream double-buffered against compute"}
+               "path": "eager calls of the C API (gb_decode_attention per layer and step); inputs copied from "
+                       "pinned host memory and outputs read back every step with cudaMemcpyAsync, on a copy "
+                       "stream double-buffered against compute"}
         status = pool.status()
         if status != 0:
             raise RuntimeError(f"device status {status} after the e2e steps: the measurement is invalid")
