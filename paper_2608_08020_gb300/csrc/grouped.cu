@@ -503,6 +503,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(ctl + kBarSchedEmpty + 8 * k);
       if (id < 0) break;
       const Unit x = load_unit(v, id);
+      // This row's record (member beam, its record slot): loaded now, used at the unit's
+      // end, so the two dependent loads complete behind the unit's tiles.
+      const int m = x.t * members_per_tile + r / G, gg = r % G;
+      const int bk = m < x.g ? v.seg_members[x.moff + m] : 0;
+      const int r_idx = v.seg_rec_off[bk] + x.sp;
       float m_ref = -INFINITY, l = 0.f;
       for (int j = 0; j < x.ntok; ++j, ++n) {
         const uint32_t sb = n % kSBufs;
@@ -602,10 +607,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(ctl + kBarXchFull);
       if (!wait_or_abort(ctl + kBarXchFull, uidx & 1, abort_flag)) break;
       const float l_all = l + xch[(slot * 2 + 1 - grp) * 128 + r];
-      const int m = x.t * members_per_tile + r / G, gg = r % G;
-      const int bk = m < x.g ? v.seg_members[x.moff + m] : 0;
       const int b = bk / kMaxSegDepth;
-      const int r_idx = v.seg_rec_off[bk] + x.sp;
       const bool has = m < x.g && r_idx < kMaxSegRecords;
       float* rec = v.grec + (((size_t)b * kMaxSegRecords + r_idx) * v.Hkv + x.h) * v.record_floats;
       // Group k writes columns [64k, 64k + 64) of the output.
