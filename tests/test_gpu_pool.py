@@ -108,3 +108,32 @@ def test_multi_layer_steps_match_oracle(cuda):
             g.probe(); o.probe(); g.prune(); o.prune()
             assert_pool_equal(g.pool.read_state(), o.pool, wl.page_size, means="tol")
     assert g.pool.status() == 0
+
+
+def test_bf16_grouped_step_out_of_pages_and_all_released(cuda):
+    """The bf16 path (grouped + per-beam kernels on two streams): a step that runs out of pages
+    changes nothing, reports GB_ERR_OOM and gives zero outputs; after every slot is released a
+    step has no work and gives zeros with the status clean."""
+    import torch
+    from workload.configs import QWEN3_8B_LAYER
+    wl = dataclasses.replace(QWEN3_8B_LAYER, beams=32, prompt_len=64, context=80, hidden=256)
+    g, o = _runs(wl, num_pages=4 + 32 + 31)       # prompt: 4 shared pages; one page per beam at L = 64
+    g.append(15)
+    o.append(15)                                  # tokens 64..78 in each beam's new page, 31 pages free
+    out = g.decode_step().cpu().numpy()
+    assert (np.abs(out) > 0).any() and g.pool.status() == 0   # token 79 still fits the page
+    o.decode_step(compute=False)
+    assert int(g.pool.read_state()["seg_cover"].sum()) > 0    # the shared prompt goes through the grouped path
+    out = g.decode_step().cpu().numpy()           # position 80 needs a new page per beam: 32 > 31 free
+    assert o.decode_step() is None
+    assert g.pool.status() == ERR_OOM == o.pool.status
+    assert (out == 0).all()
+    g.pos -= 1
+    o.pos = g.pos
+    assert_pool_equal(g.pool.read_state(), o.pool, wl.page_size, means="exact", dtype="bf16")
+    g.pool.clear_status()
+    g.pool.release(torch.arange(32, dtype=torch.int32, device=cuda))
+    out = g.decode_step().cpu().numpy()
+    assert (out == 0).all() and g.pool.status() == 0
+    st = g.pool.read_state()
+    assert not st["active"].any() and (st["refcnt"] == 0).all()
