@@ -761,6 +761,9 @@ def run_ours(args) -> None:
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = oracle_sample(wl, args.cpu_steps, args.cpu_beams)
+        one = oracle_sample(wl, max(1, args.cpu_steps // 8), 2, workers=1)   # the same oracle on one core
+        cpu["single_core"] = {"value": one["value"], "unit": one["unit"], "seconds": one["seconds"],
+                              "sample": one["sample"]}
     if rank == 0:
         line = {
             "metric": "beam-decode attn beam-tokens/s + achieved HBM TB/s vs peak; prune+branch us/step",
