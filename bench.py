@@ -596,9 +596,11 @@ def run_ours(args) -> None:
     fork_us = statistics.mean(profs[i]["fork"][0].elapsed_time(profs[i]["fork"][1]) for i in timed_rounds) * 1e3 \
         if (timed_rounds and seq is not None) else None
     grouped_on = flags != B.GB_PATH_PER_BEAM and wl.kv_dtype == "bf16" and D == 128
+    # The per-beam kernel: warp-level MMAs for bf16 pools with 128-dim heads, paired fp32 FMAs otherwise.
+    dec = "k_decode_mma" if wl.kv_dtype == "bf16" and D == 128 else "k_decode"
 
     # Algorithmic work per launch, from the library's per-step records:
-    #   k_decode:  tokens it reads (all KV heads, K and V) + the queries;
+    #   per-beam:  tokens it reads (all KV heads, K and V) + the queries;
     #   k_grouped: K/V tiles it reads (once per 128-row query tile) and the useful flops
     #              4 * D per (query row, token) for Q.K^T and P.V.
     esz = 2 if wl.kv_dtype == "bf16" else 4
@@ -621,7 +623,7 @@ def run_ours(args) -> None:
     tpeak = peaks.get("bf16_tflops_sustained") or peaks.get("bf16_tflops")
     tpeak_src = "measured sustained" if tpeak else "fallback"
     tpeak = tpeak or 1700.0
-    kernels = {"k_decode": {"us": dec_avg_s * 1e6, "bytes": dec_bytes, "gbps": achieved, "frac_hbm": achieved / peak}}
+    kernels = {dec: {"us": dec_avg_s * 1e6, "bytes": dec_bytes, "gbps": achieved, "frac_hbm": achieved / peak}}
     if grouped_on and gr_avg_s > 0:
         kernels["k_grouped"] = {"us": gr_avg_s * 1e6, "bytes": gr_bytes, "gbps": gr_bytes / gr_avg_s / 1e9,
                                 "frac_hbm": gr_bytes / gr_avg_s / 1e9 / peak, "flops": gr_flops,
@@ -629,20 +631,20 @@ def run_ours(args) -> None:
                                 "segments": statistics.mean(int(s[4]) for s in stats),
                                 "work_units": statistics.mean(int(s[5]) * Hkv for s in stats)}
     att_avg_s = statistics.mean(att_ms) / 1e3
-    dominant = "k_grouped" if "k_grouped" in kernels and gr_avg_s > dec_avg_s else "k_decode"
+    dominant = "k_grouped" if "k_grouped" in kernels and gr_avg_s > dec_avg_s else dec
     if "k_grouped" in kernels:
         # The grouped and per-beam kernels run concurrently on disjoint SMs: the pair is
         # one phase of the step, timed from before the fork to after the join.
-        tr = [captured_traffic(k, wl.name, args.flags) for k in ("k_grouped", "k_decode")]
+        tr = [captured_traffic(k, wl.name, args.flags) for k in ("k_grouped", dec)]
         pair_bytes = gr_bytes + dec_bytes
-        roofline = {"bound": "hbm", "kernel": "k_grouped + k_decode (concurrent, disjoint SMs)",
+        roofline = {"bound": "hbm", "kernel": f"k_grouped + {dec} (concurrent, disjoint SMs)",
                     "achieved": pair_bytes / att_avg_s / 1e9, "peak": peak, "unit": "GB/s",
                     "frac": pair_bytes / att_avg_s / 1e9 / peak,
                     "traffic": (tr[0] + tr[1]) if None not in tr else None, "bytes_per_launch": pair_bytes,
                     "phase_us": att_avg_s * 1e6, "peak_source": f"{peak_src} hbm_gbs"}
-    elif dominant == "k_decode":
-        roofline = {"bound": "hbm", "kernel": "k_decode (split-KV decode)", "achieved": achieved, "peak": peak,
-                    "unit": "GB/s", "frac": achieved / peak, "traffic": captured_traffic("k_decode", wl.name, args.flags), "bytes_per_launch": dec_bytes,
+    elif dominant == dec:
+        roofline = {"bound": "hbm", "kernel": f"{dec} (split-KV decode)", "achieved": achieved, "peak": peak,
+                    "unit": "GB/s", "frac": achieved / peak, "traffic": captured_traffic(dec, wl.name, args.flags), "bytes_per_launch": dec_bytes,
                     "peak_source": f"{peak_src} hbm_gbs"}
     else:
         kg = kernels["k_grouped"]

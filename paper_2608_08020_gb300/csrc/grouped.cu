@@ -652,40 +652,47 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-// 5D tensor map over the whole pool, which is viewed as rows of D = 128 bf16 (256 bytes):
+// 5D tensor maps over the whole pool, which is viewed as rows of D = 128 bf16 (256 bytes):
 // dims {64 dims, 8 rows, 2 halves of D, K|V, row groups of 8}, strides {256, 128,
-// Hkv * P * 256 (K slab to V slab), 2048} bytes, box {64, 8, 2, 1, P / 8} = K (K|V
-// coordinate 0) or V (coordinate 1) of one page of one head.  The box lands in shared
-// memory as [row group][half][8 rows][64 dims] with the 128-byte swizzle.  The row-group
-// extent ends with the last K slab, so every coordinate in range addresses a real K and
-// V slab.
-bool make_kv_tensor_map(gb_pool* pool) {
+// Hkv * P * 256 (K slab to V slab), 2048} bytes.  The grouped kernel's box {64, 8, 2, 1,
+// P / 8} is K (K|V coordinate 0) or V (coordinate 1) of one page of one head; the per-beam
+// kernel's box {64, 8, 2, 2, 2} is K and V of 16 tokens of one head.  A box lands in shared
+// memory in the dims' order ([row group][K|V][half][8 rows][64 dims]) with the 128-byte
+// swizzle.  The row-group extent ends with the last K slab, so every coordinate in range
+// addresses a real K and V slab.  Sets have_tmap (grouped) and have_dtmap (per-beam).
+void make_kv_tensor_maps(gb_pool* pool) {
   typedef CUresult (*EncodeFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
   static EncodeFn encode = nullptr;
+  pool->have_tmap = pool->have_dtmap = false;
   if (!encode) {
     cudaDriverEntryPointQueryResult qr;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", reinterpret_cast<void**>(&encode), 12000,
                                          cudaEnableDefault, &qr) != cudaSuccess ||
         qr != cudaDriverEntryPointSuccess || !encode)
-      return false;
+      return;
   }
   const PoolView& v = pool->view;
-  if (v.P % 8 != 0 || kTok % v.P != 0 || kTok / v.P > 16) return false;
+  if (v.dtype != GB_BF16 || v.D != 128) return;
   const unsigned long long rows = (unsigned long long)v.layers * v.num_pages * 2 * v.Hkv * v.P;
-  if (rows >= (1ull << 31)) return false;
+  if (rows >= (1ull << 31)) return;
   cuuint64_t dims[5] = {64, 8, 2, 2, (rows - (unsigned long long)v.Hkv * v.P) / 8};
   cuuint64_t strides[4] = {256, 128, (cuuint64_t)v.Hkv * v.P * 256, 2048};
-  cuuint32_t box[5] = {64, 8, 2, 1, (cuuint32_t)(v.P / 8)};
   cuuint32_t es[5] = {1, 1, 1, 1, 1};
-  CUtensorMap* m = reinterpret_cast<CUtensorMap*>(pool->tmap);
-  const CUresult r = encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, v.kv, dims, strides, box, es,
-                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  pool->have_tmap = r == CUDA_SUCCESS;
   pool->tmap_oob = (int)dims[4];
-  return pool->have_tmap;
+  if (v.P % 8 == 0 && kTok % v.P == 0 && kTok / v.P <= 16) {
+    cuuint32_t box[5] = {64, 8, 2, 1, (cuuint32_t)(v.P / 8)};
+    pool->have_tmap = encode(reinterpret_cast<CUtensorMap*>(pool->tmap), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, v.kv,
+                             dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
+  if (v.P % 16 == 0) {
+    cuuint32_t box[5] = {64, 8, 2, 2, 2};
+    pool->have_dtmap = encode(reinterpret_cast<CUtensorMap*>(pool->dtmap), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, v.kv,
+                              dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
 }
 
 template <int G>

@@ -122,7 +122,7 @@ __host__ __device__ inline int* plan_start(const PoolView& v, int mode) {
 }
 
 #ifndef GB_DECODE_WEIGHT
-#define GB_DECODE_WEIGHT 120  // relative cost of a per-beam token against a grouped tile token (percent)
+#define GB_DECODE_WEIGHT 60  // relative cost of a per-beam token against a grouped tile token (percent)
 #endif
 
 #ifndef GB_SPLIT_BYTES_PER_SM
@@ -266,6 +266,8 @@ struct gb_pool {
   unsigned long long seg_gen = 0;           // segment rebuilds so far
   alignas(64) unsigned char tmap[128];      // CUtensorMap over the KV pool (grouped path)
   bool have_tmap = false;
+  alignas(64) unsigned char dtmap[128];     // CUtensorMap over the KV pool (per-beam bf16 path)
+  bool have_dtmap = false;
   int tmap_oob = 0;                          // first row group past the tensor map (loads zeros)
   std::string last_error;
   unsigned long long launches = 0;          // kernels launched by this pool
@@ -308,7 +310,7 @@ cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* 
                                cudaStream_t s);
 cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s);
 cudaError_t launch_grouped(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s);
-bool make_kv_tensor_map(gb_pool* pool);
+void make_kv_tensor_maps(gb_pool* pool);
 cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
                          float bias, const uint8_t* mask, float* score_out, const float* scores_in,
                          cudaStream_t s);

@@ -536,7 +536,8 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
                64 % cfg->page_size == 0)
                   ? 1
                   : 0;
-  if (v.grouped && !make_kv_tensor_map(p)) v.grouped = 0;
+  make_kv_tensor_maps(p);
+  if (v.grouped && !p->have_tmap) v.grouped = 0;
   // The per-beam kernel of a grouped step runs on a second stream of the pool, forked from
   // and joined back into the caller's stream with two events.
   if (v.grouped && (cudaStreamCreateWithFlags(&p->aux, cudaStreamNonBlocking) != cudaSuccess ||
