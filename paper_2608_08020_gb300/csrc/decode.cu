@@ -454,9 +454,19 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 // about a hundred, which is what bounds the per-beam kernel when it shares the GPU with
 // the grouped kernel.
 constexpr int kMmaStageBytes = 2 * kChunk * 128 * 2;  // K and V of 16 tokens x 128 bf16
+#ifndef GB_MMA_WARPS
+#define GB_MMA_WARPS 12  // warps per CTA of k_decode_mma (one CTA per SM)
+#endif
+#ifndef GB_MMA_STAGES
+#define GB_MMA_STAGES 2  // ring depth per warp
+#endif
+#ifndef GB_MMA_CHAINS
+#define GB_MMA_CHAINS 2  // independent accumulator chains of the 8 S^T MMAs of a chunk
+#endif
+constexpr int kMmaWarps = GB_MMA_WARPS, kMmaStages = GB_MMA_STAGES, kMmaChains = GB_MMA_CHAINS;
 struct DecodeMmaSmem {
-  static constexpr int STAGES = kDecodeWarps * kDecodeStages * kMmaStageBytes;
-  static constexpr int BARS = kDecodeWarps * kDecodeStages * 8;
+  static constexpr int STAGES = kMmaWarps * kMmaStages * kMmaStageBytes;
+  static constexpr int BARS = kMmaWarps * kMmaStages * 8;
   static constexpr int PLAN_BYTES = 3 * (kMaxBeams + 1) * 4;
   static constexpr int TOTAL = 1024 + STAGES + BARS + PLAN_BYTES;  // 1024: alignment slack
   static_assert(TOTAL <= 232448, "shared memory per block");
@@ -507,7 +517,7 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 }
 
 template <int G>
-__global__ void __launch_bounds__(kDecodeWarps * 32, 1)
+__global__ void __launch_bounds__(kMmaWarps * 32, 1)
     k_decode_mma(PoolView v, const __grid_constant__ CUtensorMap tm, int layer, const __nv_bfloat16* __restrict__ q,
                  float qscale, int mode, int W) {
   pdl_wait();
@@ -521,9 +531,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
   int* s_start = s_n + (kMaxBeams + 1);
   if (v.ctl[kCtlStepOk] == 0) return;
   if (mode == 1) {  // beside the grouped kernel: this kernel's share of the SMs (decode_ctas)
-    const int nd = decode_ctas(v, W / kDecodeWarps);
+    const int nd = decode_ctas(v, W / kMmaWarps);
     if ((int)blockIdx.x >= nd) return;
-    W = nd * kDecodeWarps;
+    W = nd * kMmaWarps;
   }
   {
     const int* off = plan_off(v, mode);
@@ -539,18 +549,18 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = lane >> 2, c = lane & 3;  // MMA fragment row (token / dim) and column pair (heads 2c, 2c + 1)
-  const uint32_t stage0 = smem_addr(smem) + warp * kDecodeStages * kMmaStageBytes;
-  const uint32_t bar0 = smem_addr(smem) + S::STAGES + warp * kDecodeStages * 8;
+  const uint32_t stage0 = smem_addr(smem) + warp * kMmaStages * kMmaStageBytes;
+  const uint32_t bar0 = smem_addr(smem) + S::STAGES + warp * kMmaStages * 8;
 
   const int Tot = s_off[v.max_beams];
-  const int w = blockIdx.x * kDecodeWarps + warp;
+  const int w = blockIdx.x * kMmaWarps + warp;
   const int cw = (Tot + W - 1) / W;
   const int x_begin = w * cw;
   const int x_end = min(Tot, x_begin + cw);
   if (x_begin >= x_end) return;
 
   if (lane == 0) {
-    for (int s = 0; s < kDecodeStages; ++s) mbar_init(bar0 + 8 * s, 1);
+    for (int s = 0; s < kMmaStages; ++s) mbar_init(bar0 + 8 * s, 1);
     fence_mbar_init();
   }
   __syncwarp();
@@ -580,6 +590,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     }
     return __shfl_sync(0xffffffffu, pw_lane, qi.i - pw_i0);
   };
+  // Row group of a chunk's first K row: the whole pool has fewer than 2^31 rows (a condition
+  // of the tensor map), so 32-bit arithmetic is exact; P is 16, 32 or 64.
+  const int pg8 = v.P >> 3, layer_pages = layer * v.num_pages;
   auto issue = [&](const ChunkIter& qi, int page, int stage) {
     if (lane == 0) {
       if (page < 0 || page >= v.num_pages) {
@@ -587,8 +600,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         page = 0;
       }
       const int tok = qi.tok0 + qi.i * kChunk;
-      const long long slab = (((long long)layer * v.num_pages + page) * 2) * v.Hkv + qi.h;
-      const int wrow = (int)((slab * v.P + tok % v.P) / 8);
+      const int wrow = ((layer_pages + page) * 2 * v.Hkv + qi.h) * pg8 + ((tok & (v.P - 1)) >> 3);
       const uint32_t bar = bar0 + 8 * stage;
       mbar_arrive_expect_tx(bar, kMmaStageBytes);
       tma_chunk(stage0 + stage * kMmaStageBytes, &tm, wrow, bar, pol);
@@ -598,7 +610,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
   ChunkIter ip = it;
   int ip_x = x_begin;
   int ip_page = load_page(ip);
-  for (int s = 0; s < kDecodeStages; ++s) {
+  for (int s = 0; s < kMmaStages; ++s) {
     if (ip_x < x_end) {
       issue(ip, ip_page, s);
       ++ip_x;
@@ -629,6 +641,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
   int L = 0;
   bool fresh = true;
 
+  int stage = 0;
+  uint32_t parity = 0;
   for (int x = x_begin, k = 0; x < x_end; ++x, ++k) {
     if (fresh) {
       L = v.seq_len[it.b];
@@ -644,13 +658,11 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
       l0 = l1 = 0.f;
       fresh = false;
     }
-    const int stage = k % kDecodeStages;
-    const uint32_t parity = (k / kDecodeStages) & 1;
     if (!mbar_wait_bounded(bar0 + 8 * stage, parity, kWaitLimitNs)) {
       if (lane == 0) set_status(v.ctl, GB_ERR_TIMEOUT);
-      for (int s = 0; s < kDecodeStages; ++s) {
+      for (int s = 0; s < kMmaStages; ++s) {
         const int kk = k + s;
-        if (x + s < ip_x) mbar_wait_bounded(bar0 + 8 * (kk % kDecodeStages), (kk / kDecodeStages) & 1, kWaitLimitNs / 4);
+        if (x + s < ip_x) mbar_wait_bounded(bar0 + 8 * (kk % kMmaStages), (kk / kMmaStages) & 1, kWaitLimitNs / 4);
       }
       return;
     }
@@ -658,18 +670,24 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
     const int tok0 = it.tok0 + it.i * kChunk;
     const int nvalid = min(kChunk, L - tok0);  // >= 1: a chunk starts before the beam's length
 
-    // ---- S^T = K . Q^T (two accumulator chains) ------------------------------
-    float sa[4] = {0.f, 0.f, 0.f, 0.f}, sbk[4] = {0.f, 0.f, 0.f, 0.f};
+    // ---- S^T = K . Q^T (kMmaChains independent accumulator chains) -----------
+    float sacc[kMmaChains][4];
+#pragma unroll
+    for (int ch = 0; ch < kMmaChains; ++ch) sacc[ch][0] = sacc[ch][1] = sacc[ch][2] = sacc[ch][3] = 0.f;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       uint32_t a0, a1, a2, a3;
       ldsm_x4(sb + koff[j & 3] + (j >> 2) * 1024, a0, a1, a2, a3);
-      if (j & 1) mma_bf16(sbk, a0, a1, a2, a3, qf[j][0], qf[j][1]);
-      else mma_bf16(sa, a0, a1, a2, a3, qf[j][0], qf[j][1]);
+      mma_bf16(sacc[j % kMmaChains], a0, a1, a2, a3, qf[j][0], qf[j][1]);
     }
     float sc[4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) sc[e] = (sa[e] + sbk[e]) * qscale;
+    for (int e = 0; e < 4; ++e) {
+      float t = sacc[0][e];
+#pragma unroll
+      for (int ch = 1; ch < kMmaChains; ++ch) t += sacc[ch][e];
+      sc[e] = t * qscale;
+    }
     if (nvalid < kChunk) {
       // Tokens past the beam's length: no score, and zero V rows (the page's rows there
       // hold whatever the pool held), so that 0 * V stays 0 in the MMA.
@@ -730,6 +748,10 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
         ip_page = load_page(ip);
       }
     }
+    if (++stage == kMmaStages) {
+      stage = 0;
+      parity ^= 1u;
+    }
     const bool last_of_bh = (it.i == it.n - 1) || (x + 1 == x_end);
     if (last_of_bh) {
 #pragma unroll
@@ -773,7 +795,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 // Beams with more than kCombineCache records take the scale factors from global memory.
 constexpr int kCombineCache = 128;
 
-__global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, float* __restrict__ out) {
+__global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, int wpc, float* __restrict__ out) {
   pdl_wait();
   pdl_launch_dependents();
   __shared__ float s_m[kCombineCache * 8], s_l[kCombineCache * 8];
@@ -790,7 +812,7 @@ __global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, fl
     return;
   }
   const int Tot = plan_off(v, mode)[v.max_beams];
-  if (mode == 1) W = decode_ctas(v, W / kDecodeWarps) * kDecodeWarps;  // the warps the decode kernel used
+  if (mode == 1) W = decode_ctas(v, W / wpc) * wpc;  // the warps the decode kernel used (wpc per CTA)
   const int c = Tot > 0 ? (Tot + W - 1) / W : 1;
   const int off = plan_off(v, mode)[b] + h * n;
   const int first = off / c, npb = n > 0 ? (off + n - 1) / c - first + 1 : 0;  // per-beam records
@@ -888,19 +910,21 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  const int W = pool->decode_warps;
+  int W = pool->decode_warps, wpc = kDecodeWarps;  // warps launched, warps per CTA (one CTA per SM)
   const float qscale = scale * 1.4426950408889634f;  // log2(e): softmax in base 2
   prof_begin(pool, GB_PROF_DECODE, sd);
   cudaError_t e;
   if constexpr (DT == GB_BF16) {
-    if (pool->have_dtmap) {
+    if (pool->have_dtmap && pool->num_sms * kMmaWarps <= kMaxDecodeWarps) {
       static bool mma_configured = false;
       if (!mma_configured) {
         e = cudaFuncSetAttribute(k_decode_mma<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeMmaSmem::TOTAL);
         if (e != cudaSuccess) return e;
         mma_configured = true;
       }
-      e = launch_pdl(k_decode_mma<G>, W / kDecodeWarps, kDecodeWarps * 32, DecodeMmaSmem::TOTAL, sd, pool->view,
+      wpc = kMmaWarps;
+      W = pool->num_sms * kMmaWarps;  // one CTA per SM, as the grouped kernel's split assumes
+      e = launch_pdl(k_decode_mma<G>, W / kMmaWarps, kMmaWarps * 32, DecodeMmaSmem::TOTAL, sd, pool->view,
                      *reinterpret_cast<const CUtensorMap*>(pool->dtmap), layer, static_cast<const __nv_bfloat16*>(q),
                      qscale, mode, W);
     } else {
@@ -920,7 +944,7 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
   }
   prof_end(pool, GB_PROF_ATTENTION, s);
   prof_begin(pool, GB_PROF_COMBINE, s);
-  e = launch_pdl(k_combine, pool->view.max_beams * pool->view.Hkv, 128, 0, s, pool->view, mode, W, out);
+  e = launch_pdl(k_combine, pool->view.max_beams * pool->view.Hkv, 128, 0, s, pool->view, mode, W, wpc, out);
   prof_end(pool, GB_PROF_COMBINE, s);
   pool->launches += 2;
   return e;
@@ -942,7 +966,7 @@ static cudaError_t launch_view_t(const PoolView& v, int W, int layer, const void
   k_decode<DT, G><<<W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s>>>(v, layer, q, qscale, 0, W);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_combine<<<v.max_beams * v.Hkv, 128, 0, s>>>(v, 0, W, out);
+  k_combine<<<v.max_beams * v.Hkv, 128, 0, s>>>(v, 0, W, kDecodeWarps, out);
   return cudaGetLastError();
 }
 
