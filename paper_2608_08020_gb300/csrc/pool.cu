@@ -345,8 +345,9 @@ __global__ void k_append(PoolView v, int layer, int n_tokens, const char* kin, c
   // Rows differ from every row written below, so both loops run concurrently.
   const int ncow = v.ctl[kCtlCowJobs];
   const long long per_job = 2LL * v.Hkv * v.P * vec_per_row;
-  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < per_job * ncow;
-       i += (long long)gridDim.x * blockDim.x) {
+  const long long nthreads = (long long)gridDim.x * gridDim.y * blockDim.x;
+  for (long long i = ((long long)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x; i < per_job * ncow;
+       i += nthreads) {
     const int j = (int)(i / per_job);
     long long r = i % per_job;
     const int vec = (int)(r % vec_per_row); r /= vec_per_row;
@@ -358,26 +359,25 @@ __global__ void k_append(PoolView v, int layer, int n_tokens, const char* kin, c
     uint4* dst = reinterpret_cast<uint4*>(v.kv + kv_elem_offset(v, layer, v.cow[3 * j + 1], kv, head, row) * v.esize);
     dst[vec] = src[vec];
   }
-  const long long per_tok = (long long)v.max_beams * v.Hkv * vec_per_row;
-  const long long total = per_tok * n_tokens * 2;
-  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
-       i += (long long)gridDim.x * blockDim.x) {
-    const int kv = (int)(i / (per_tok * n_tokens));
-    long long r = i % (per_tok * n_tokens);
-    const int k = (int)(r / per_tok);
-    r %= per_tok;
-    const int vec = (int)(r % vec_per_row);
-    r /= vec_per_row;
-    const int head = (int)(r % v.Hkv);
-    const int b = (int)(r / v.Hkv);
-    if (!v.active[b]) continue;
-    const int pos = v.seq_len[b] - n_tokens + k;
-    if (pos < 0) continue;
-    const int page = v.tables[(size_t)b * v.max_pages + pos / v.P];
-    if (page < 0 || page >= v.num_pages) { set_status(v.ctl, GB_ERR_INVALID); continue; }
-    const char* src = (kv ? vin : kin) + ((((long long)k * v.max_beams + b) * v.Hkv + head) * v.D) * v.esize;
-    char* dst = v.kv + kv_elem_offset(v, layer, page, kv, head, pos % v.P) * v.esize;
-    reinterpret_cast<uint4*>(dst)[vec] = reinterpret_cast<const uint4*>(src)[vec];
+  // New rows: blockIdx.y walks (K|V, token), x covers (slot, head, 16-byte vector) with
+  // 32-bit index arithmetic (a row is 256 bytes, 16 vectors, for every supported shape).
+  const int per_tok = v.max_beams * v.Hkv * vec_per_row;
+  for (int y = blockIdx.y; y < 2 * n_tokens; y += gridDim.y) {
+    const int kv = y >= n_tokens ? 1 : 0;
+    const int k = y - kv * n_tokens;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < per_tok; i += gridDim.x * blockDim.x) {
+      const int vec = i & 15;
+      const int r = i >> 4;
+      const int b = r / v.Hkv, head = r - b * v.Hkv;
+      if (!v.active[b]) continue;
+      const int pos = v.seq_len[b] - n_tokens + k;
+      if (pos < 0) continue;
+      const int page = v.tables[(size_t)b * v.max_pages + pos / v.P];
+      if (page < 0 || page >= v.num_pages) { set_status(v.ctl, GB_ERR_INVALID); continue; }
+      const char* src = (kv ? vin : kin) + ((((long long)k * v.max_beams + b) * v.Hkv + head) * v.D) * v.esize;
+      char* dst = v.kv + kv_elem_offset(v, layer, page, kv, head, pos % v.P) * v.esize;
+      reinterpret_cast<uint4*>(dst)[vec] = reinterpret_cast<const uint4*>(src)[vec];
+    }
   }
 }
 
@@ -609,7 +609,8 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
   if (layer != pool->next_layer) return fail(pool, GB_ERR_STATE, "layers of a step must be called in order");
   if (layer == 0) {
     prof_begin(pool, GB_PROF_PLAN, s);
-    launch_pdl(k_step_begin, 1, 1024, 0, s, pool->view, n_tokens,
+    // One thread per slot (rounded up to a warp): the planner's block scans span only the pool's slots.
+    launch_pdl(k_step_begin, 1, std::max(32, (pool->cfg.max_beams + 31) / 32 * 32), 0, s, pool->view, n_tokens,
                pool->view.grouped ? pool->view.seg_cover : nullptr);
     prof_end(pool, GB_PROF_PLAN, s);
     pool->launches += 1;
@@ -619,11 +620,10 @@ static gb_status append_layer(gb_pool* pool, int layer, int n_tokens, const void
   } else if (n_tokens != pool->step_tokens) {
     return fail(pool, GB_ERR_STATE, "token count differs from the one layer 0 reserved");
   }
-  const long long vecs = 2LL * n_tokens * pool->cfg.max_beams * pool->cfg.num_kv_heads *
-                         (pool->view.D * pool->view.esize / 16);
-  const int grid = (int)std::min<long long>((vecs + 255) / 256, pool->num_sms * 8LL);
+  const int per_tok = pool->cfg.max_beams * pool->cfg.num_kv_heads * (pool->view.D * pool->view.esize / 16);
+  const dim3 grid(std::max(1, std::min((per_tok + 255) / 256, pool->num_sms * 8)), std::min(2 * n_tokens, 65535));
   prof_begin(pool, GB_PROF_APPEND, s);
-  launch_pdl(k_append, std::max(grid, 1), 256, 0, s, pool->view, layer, n_tokens, static_cast<const char*>(k),
+  launch_pdl(k_append, grid, 256, 0, s, pool->view, layer, n_tokens, static_cast<const char*>(k),
              static_cast<const char*>(v));
   prof_end(pool, GB_PROF_APPEND, s);
   pool->launches += 1;
