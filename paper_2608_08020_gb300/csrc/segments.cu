@@ -118,6 +118,10 @@ __global__ void k_seg_members(PoolView v) {
   if (slot < v.seg_g[id] && v.seg_mem_off[id] + slot < cap) v.seg_members[v.seg_mem_off[id] + slot] = idx;
 }
 
+#ifndef GB_SEG_UNITS_PCT
+#define GB_SEG_UNITS_PCT 200  // grouped work units aimed at per multiprocessor, in percent
+#endif
+
 // One CTA: the grouped work list.  Each segment has ceil(g*G/128) query tiles; each
 // tile is split along the segment's tokens into pieces of `split` tokens (a multiple of
 // the grouped kernel's 128-token K/V tile) so that the list has about two units per
@@ -146,7 +150,7 @@ __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
   }
   if (threadIdx.x == 0) {
     const long long work = (long long)tiletok * v.Hkv;              // tile-tokens over all heads
-    const long long target_units = 2LL * (v.num_sms > 0 ? v.num_sms : 1);
+    const long long target_units = (long long)GB_SEG_UNITS_PCT * (v.num_sms > 0 ? v.num_sms : 1) / 100;
     int split = (int)(((work + target_units - 1) / target_units + 127) / 128 * 128);
     const int max_tokens = v.max_pages * v.P;
     const int min_split = ((max_tokens + (kMaxSegRecords - kMaxSegDepth) - 1) / (kMaxSegRecords - kMaxSegDepth) + 127) /
