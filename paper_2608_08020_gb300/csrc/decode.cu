@@ -7,14 +7,14 @@
 // (beam, kv-head, 16-token chunk) units, ordered beam-major.  Every warp of a
 // persistent grid takes one contiguous range of that list, so work is
 // balanced to within one chunk whatever the beams' lengths.  A warp streams
-// its chunks through a private ring of shared-memory stages filled by 1D
-// bulk copies (TMA): one 4 KiB K slab and one 4 KiB V slab per chunk, both
-// contiguous in a page.  When its range leaves a (beam, head) it writes an
-// unnormalised partial (m, l, o) for the G query heads of that KV head; the
-// combine kernel merges the partials of each (beam, head) with the standard
-// log-sum-exp rule.
+// its chunks through a private ring of shared-memory stages filled by TMA.
+// When its range leaves a (beam, head) it writes an unnormalised partial
+// (m, l, o) for the G query heads of that KV head; the combine kernel merges
+// the partials of each (beam, head) with the standard log-sum-exp rule.
 //
-// Lane layout inside a warp: 4 token rows x 8 lanes.  Lane j of row r owns
+// k_decode fills a stage with two 1D bulk copies (one 4 KiB K slab and one
+// 4 KiB V slab per chunk, both contiguous in a page).  Its lane layout inside
+// a warp: 4 token rows x 8 lanes.  Lane j of row r owns
 // two 16-byte pieces of every token row (bytes [16j, 16j+16) and
 // [128+16j, 128+16j+16) of the 256-byte row), i.e. 16 bf16 or 8 fp32 dims,
 // and handles tokens r, r+4, r+8, r+12 of a chunk.  Scores are reduced with
@@ -451,8 +451,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 // state and every rescale stay inside the lane.  Base-2 softmax; the running max is raised
 // only when a chunk's max exceeds it by more than 8 (p <= 2^8 otherwise).  This cuts the
 // per-chunk work of a warp from ~700 instructions per lane (k_decode's paired FMAs) to
-// about a hundred, which is what bounds the per-beam kernel when it shares the GPU with
-// the grouped kernel.
+// ~250-300 warp instructions, which is what bounds the per-beam kernel when it shares the
+// GPU with the grouped kernel; 12 warps per SM with 2-stage rings hide more of each
+// warp's instruction latency than 8 warps with 3 stages, in the same shared memory.
 constexpr int kMmaStageBytes = 2 * kChunk * 128 * 2;  // K and V of 16 tokens x 128 bf16
 #ifndef GB_MMA_WARPS
 #define GB_MMA_WARPS 12  // warps per CTA of k_decode_mma (one CTA per SM)
