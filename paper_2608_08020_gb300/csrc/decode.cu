@@ -787,20 +787,15 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 1)
 // Merge the partial records of each (beam, kv head) into out[b][h*G+g][:]: the split-KV
 // records of the warps that covered the beam's per-beam range and, in mode 1, the grouped
 // records of the beam's shared-prefix segments (the log-sum-exp merge, base 2).
-// One CTA of 128 threads per (beam, kv head), built so that many loads are in flight:
-//   1. the (m, l) pairs of all records go to shared memory in one sweep;
-//   2. warp w takes query heads g = w, w + 4: M_g = max m, the scale factors
-//      2^(m - M_g) (kept in place of m) and L_g = sum l * 2^(m - M_g);
-//   3. every thread takes 4 consecutive output elements and sums the records 8 at a
-//      time with float4 loads, then divides by L_g.
-// Beams with more than kCombineCache records take the scale factors from global memory.
-constexpr int kCombineCache = 128;
-
+// One CTA of 128 threads per (beam, kv head); thread t owns 4 consecutive output elements
+// of one query head g and folds all records in one pass, 8 records of loads in flight at a
+// time: M = running max of the records' m, acc = sum o * 2^(m - M), L = sum l * 2^(m - M),
+// rescaled when M rises.  Every thread of a warp reads the same (m, l) words (one head per
+// warp at D = 128, two at D = 64), so those loads are broadcasts; the o loads are float4
+// and coalesced.
 __global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, int wpc, float* __restrict__ out) {
   pdl_wait();
   pdl_launch_dependents();
-  __shared__ float s_m[kCombineCache * 8], s_l[kCombineCache * 8];
-  __shared__ float s_M[8], s_L[8];
   const int bh = blockIdx.x;
   const int b = bh / v.Hkv, h = bh % v.Hkv;
   const int G = v.G, D = v.D, GD = G * D;
@@ -824,71 +819,51 @@ __global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, in
   auto rec_at = [&](int r) -> const float* {
     return r < npb ? prec + (size_t)r * v.record_floats : grec + (size_t)(r - npb) * gstride;
   };
-  const bool cached = R <= kCombineCache;
-  if (cached) {
-    for (int idx = threadIdx.x; idx < R * G; idx += blockDim.x) {
-      const int r = idx / G, g = idx - r * G;
-      const float* rec = rec_at(r);
-      s_m[r * 8 + g] = rec[GD + g];
-      s_l[r * 8 + g] = rec[GD + G + g];
-    }
-    __syncthreads();
-  }
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int g = warp; g < G; g += 4) {
-    float M = -INFINITY;
-    for (int r = lane; r < R; r += 32) M = fmaxf(M, cached ? s_m[r * 8 + g] : rec_at(r)[GD + g]);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    float L = 0.f;
-    for (int r = lane; r < R; r += 32) {
-      const float m = cached ? s_m[r * 8 + g] : rec_at(r)[GD + g];
-      const float l = cached ? s_l[r * 8 + g] : rec_at(r)[GD + G + g];
-      const float sc = m == -INFINITY ? 0.f : exp2f(m - M);  // a record that saw no token adds nothing
-      L = fmaf(l, sc, L);
-      if (cached) s_m[r * 8 + g] = sc;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-    if (lane == 0) {
-      s_M[g] = M;
-      s_L[g] = L;
-    }
-  }
-  __syncthreads();
   const bool vec_out = (reinterpret_cast<uintptr_t>(ob) & 15) == 0;
   for (int e4 = threadIdx.x; e4 < GD / 4; e4 += blockDim.x) {
     const int g = (e4 * 4) / D;
+    float M = -INFINITY, L = 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int r0 = 0; r0 < R; r0 += 8) {
       float4 x[8];
-      float sc[8];
+      float mk[8], lk[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
         const int r = r0 + k;
         if (r < R) {
           const float* rec = rec_at(r);
           x[k] = *reinterpret_cast<const float4*>(rec + 4 * e4);
-          if (cached) {
-            sc[k] = s_m[r * 8 + g];
-          } else {
-            const float m = rec[GD + g];
-            sc[k] = m == -INFINITY ? 0.f : exp2f(m - s_M[g]);
-          }
+          mk[k] = rec[GD + g];
+          lk[k] = rec[GD + G + g];
         } else {
           x[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-          sc[k] = 0.f;
+          mk[k] = -INFINITY;  // a record that saw no token (or none at all) adds nothing
+          lk[k] = 0.f;
         }
+      }
+      float mnew = M;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) mnew = fmaxf(mnew, mk[k]);
+      if (mnew == -INFINITY) continue;
+      if (mnew > M) {  // M = -inf the first time: acc and L are still 0
+        const float a = M == -INFINITY ? 0.f : exp2f(M - mnew);
+        acc.x *= a;
+        acc.y *= a;
+        acc.z *= a;
+        acc.w *= a;
+        L *= a;
+        M = mnew;
       }
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
-        acc.x = fmaf(x[k].x, sc[k], acc.x);
-        acc.y = fmaf(x[k].y, sc[k], acc.y);
-        acc.z = fmaf(x[k].z, sc[k], acc.z);
-        acc.w = fmaf(x[k].w, sc[k], acc.w);
+        const float sc = mk[k] == -INFINITY ? 0.f : exp2f(mk[k] - M);
+        acc.x = fmaf(x[k].x, sc, acc.x);
+        acc.y = fmaf(x[k].y, sc, acc.y);
+        acc.z = fmaf(x[k].z, sc, acc.z);
+        acc.w = fmaf(x[k].w, sc, acc.w);
+        L = fmaf(lk[k], sc, L);
       }
     }
-    const float L = s_L[g];
     const float4 res = make_float4(acc.x / L, acc.y / L, acc.z / L, acc.w / L);
     if (vec_out) {
       *reinterpret_cast<float4*>(ob + 4 * e4) = res;
