@@ -3,7 +3,7 @@
 prefixes beside the per-beam kernel) and on the per-beam path, against the oracle: an
 unaligned prompt (copy-on-write of the shared tail page), ragged tails, forks by real
 tournament rounds.  The per-beam kernel's MMA fragments hold G heads in 8 columns and its
-TMA coordinates depend on P, so each shape is a distinct case."""
+TMA coordinates depend on P and on the layer, so each shape is a distinct case."""
 import dataclasses
 
 import pytest
@@ -16,11 +16,12 @@ from workload.configs import QWEN3_8B_LAYER
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("Hq,Hkv,P", [(4, 2, 16), (16, 2, 16), (8, 1, 32), (32, 8, 64), (16, 2, 64)])
+@pytest.mark.parametrize("Hq,Hkv,P,layers", [(4, 2, 16, 1), (16, 2, 16, 1), (8, 1, 32, 1), (32, 8, 64, 1),
+                                             (16, 2, 64, 1), (32, 8, 16, 3)])
 @pytest.mark.parametrize("flags", ["auto", "per_beam"])
-def test_bf16_shapes_match_oracle(cuda, Hq, Hkv, P, flags):
+def test_bf16_shapes_match_oracle(cuda, Hq, Hkv, P, layers, flags):
     from workload.driver import GpuRun
-    wl = dataclasses.replace(QWEN3_8B_LAYER, num_q_heads=Hq, num_kv_heads=Hkv, page_size=P, beams=8,
+    wl = dataclasses.replace(QWEN3_8B_LAYER, num_layers=layers, num_q_heads=Hq, num_kv_heads=Hkv, page_size=P, beams=8,
                              prompt_len=72, context=72 + 3 * P + 40, interval=P + 24, K=4, hidden=256)
     path = B.GB_PATH_AUTO if flags == "auto" else B.GB_PATH_PER_BEAM
     g, o = GpuRun(wl), OracleRun(wl, literal_kv=True)
