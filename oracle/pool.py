@@ -8,7 +8,7 @@ What the paper fixes (Section 3.1, the paragraph after Eq. 3; Section 3.2):
 * the active count stays C (zero-sum).
 
 What this model adds, as the definition the CUDA pool must reproduce bit for
-bit (each a reading listed in the design doc):
+bit (each a reading of a passage where the paper is silent):
 
 * a page holds ``P`` consecutive token positions of one beam's context for
   every layer; a slot's block table lists its pages in position order;

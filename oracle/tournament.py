@@ -11,7 +11,7 @@ routing cases of Section 3.1:
 * Case 2, at capacity (N = C, Eq. 3): prune the bottom ``K`` and branch the
   top ``K``; pruning and branching are paired so |T_act| stays C.
 
-Readings where the paper is silent (each listed in the design doc):
+Readings where the paper is silent:
 
 * ties in the ranking keep ascending slot order (the lower slot ranks
   higher), +0 and -0 compare equal, and a NaN mean ranks after every number;
