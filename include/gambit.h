@@ -319,17 +319,22 @@ gb_status gb_pool_launch_count(gb_pool* pool, uint64_t* count);
  *   tables:  int32 [num_beams][max_pages_per_beam];  seq_len: int32 [num_beams]
  *   q:       [num_beams][num_q_heads][head_dim] in kv_dtype, 16-byte aligned
  *   out:     fp32 [num_beams][num_q_heads][head_dim]
- * Page ids are trusted: an id outside [0, num_pages) is not dereferenced (page 0 is
- * read in its place) and that row's output is unspecified.
+ * Rows must satisfy 0 <= seq_len[b] <= max_pages_per_beam * page_size: a row outside
+ * that range is not read (its output is zero) and the call's device status records
+ * GB_ERR_INVALID.  Page ids are checked too: an id outside [0, num_pages) is not
+ * dereferenced (page 0 is read in its place), that row's output is unspecified and the
+ * status records GB_ERR_INVALID.  A bounded device-side wait that runs out records
+ * GB_ERR_TIMEOUT.  gb_paged_decode_noalloc_status() reads that status word.
  *
  * The scratch array is shared by every call on a device and keeps the last call's
  * contents; each call rewrites all of it that it reads, and clears its own status
- * word.  Calls whose GPU work overlaps (different streams, or host threads issuing
+ * word first.  Calls whose GPU work overlaps (different streams, or host threads issuing
  * concurrently) race on it: keep them ordered, e.g. on one stream.
  * The first call on a device looks up the array's device address with
  * cudaGetSymbolAddress (with that device current); that first call should come
  * before any stream capture.
- * Errors: GB_ERR_INVALID for bad shapes or null/misaligned pointers,
+ * Errors: GB_ERR_INVALID for bad shapes or null/misaligned pointers, or when
+ * num_beams x ceil(max_pages_per_beam x page_size / 16) x num_kv_heads reaches 2^31,
  * GB_ERR_UNSUPPORTED for a (kv_dtype, head_dim, Hq/Hkv) without a kernel, and
  * GB_ERR_TOO_LARGE when the scratch needed, 256-byte rounded
  *   128 + 4*num_beams + 12*(num_beams+1) + 4*(W + num_beams*num_kv_heads)*G*(head_dim+2)
@@ -354,6 +359,16 @@ typedef struct {
   float scale;
 } gb_paged_decode_args;
 gb_status gb_paged_decode_noalloc(const gb_paged_decode_args* args, gb_stream_t stream);
+
+/*
+ * Device status of the most recent gb_paged_decode_noalloc() call on the current device
+ * (GB_OK, or the first error its kernels recorded: GB_ERR_INVALID for a row length or
+ * page id out of range, GB_ERR_TIMEOUT for a bounded wait that ran out).  Synchronises
+ * `stream` (pass the stream of that call) and copies the status word of the library's
+ * scratch array into *device_status with one cudaMemcpyAsync; allocates nothing.  The
+ * paper has no counterpart: it belongs to the allocation-free entry point above.
+ */
+gb_status gb_paged_decode_noalloc_status(int* device_status, gb_stream_t stream);
 
 /*
  * Apply a tournament decided on another pool (for example the generator's pool's

@@ -27,7 +27,7 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
            "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
-           "gb_paged_decode_noalloc", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_score_mlp", "gb_fork_slots", "gb_scorer_sizes", "gb_scorer_seed",
+           "gb_paged_decode_noalloc", "gb_paged_decode_noalloc_status", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_score_mlp", "gb_fork_slots", "gb_scorer_sizes", "gb_scorer_seed",
            "gb_scorer_step", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
 GB_PROF_PLAN, GB_PROF_APPEND, GB_PROF_COMBINE, GB_PROF_ATTENTION = 4, 5, 6, 7
@@ -91,6 +91,7 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_pool_set_profile_events": [V, I, V, V],
         "gb_pool_launch_count": [V, P],
         "gb_paged_decode_noalloc": [P, V],
+        "gb_paged_decode_noalloc_status": [P, V],
         "gb_pool_read_step_stats": [V, P, I, P, V],
         "gb_pool_set_capacity": [V, I],
         "gb_score_mlp": [V, V, I, V, V, V, F, I, V, V, V],
@@ -280,6 +281,14 @@ def gb_paged_decode_noalloc(args: GbPagedDecodeArgs, stream=None) -> None:
     """Paged decode attention with the library's fixed scratch (no allocation, no workspace)."""
     _check(None, load().gb_paged_decode_noalloc(ctypes.byref(args), stream_handle(stream)),
            "gb_paged_decode_noalloc")
+
+
+def gb_paged_decode_noalloc_status(stream=None) -> int:
+    """Device status of the last gb_paged_decode_noalloc call on the current device (synchronises)."""
+    st = ctypes.c_int()
+    _check(None, load().gb_paged_decode_noalloc_status(ctypes.byref(st), stream_handle(stream)),
+           "gb_paged_decode_noalloc_status")
+    return st.value
 
 
 def gb_last_error(pool: int) -> str:

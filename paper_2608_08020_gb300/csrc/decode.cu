@@ -880,11 +880,9 @@ template <int DT, int G>
 static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
                                    cudaStream_t s, cudaStream_t sd) {
   using S = DecodeSmem<DT, G>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(k_decode<DT, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, S::TOTAL);
+  {
+    const cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_decode<DT, G>), S::TOTAL);
     if (e != cudaSuccess) return e;
-    configured = true;
   }
   int W = pool->decode_warps, wpc = kDecodeWarps;  // warps launched, warps per CTA (one CTA per SM)
   const float qscale = scale * 1.4426950408889634f;  // log2(e): softmax in base 2
@@ -892,12 +890,8 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
   cudaError_t e;
   if constexpr (DT == GB_BF16) {
     if (pool->have_dtmap && pool->num_sms * kMmaWarps <= kMaxDecodeWarps) {
-      static bool mma_configured = false;
-      if (!mma_configured) {
-        e = cudaFuncSetAttribute(k_decode_mma<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, DecodeMmaSmem::TOTAL);
-        if (e != cudaSuccess) return e;
-        mma_configured = true;
-      }
+      e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_decode_mma<G>), DecodeMmaSmem::TOTAL);
+      if (e != cudaSuccess) return e;
       wpc = kMmaWarps;
       W = pool->num_sms * kMmaWarps;  // one CTA per SM, as the grouped kernel's split assumes
       e = launch_pdl(k_decode_mma<G>, W / kMmaWarps, kMmaWarps * 32, DecodeMmaSmem::TOTAL, sd, pool->view,
@@ -932,11 +926,9 @@ template <int DT, int G>
 static cudaError_t launch_view_t(const PoolView& v, int W, int layer, const void* q, float scale, float* out,
                                  cudaStream_t s) {
   using S = DecodeSmem<DT, G>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(k_decode<DT, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, S::TOTAL);
+  {
+    const cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_decode<DT, G>), S::TOTAL);
     if (e != cudaSuccess) return e;
-    configured = true;
   }
   const float qscale = scale * 1.4426950408889634f;
   k_decode<DT, G><<<W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s>>>(v, layer, q, qscale, 0, W);

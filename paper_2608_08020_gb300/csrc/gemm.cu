@@ -163,11 +163,9 @@ int gemm_splits(int M, int N, int K, int num_sms, size_t max_floats) {
 
 cudaError_t gemm_partials(const void* A, int M, const void* B, int N, int K, int splits, float* P, int* ctl,
                           cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_partials, cudaFuncAttributeMaxDynamicSharedMemorySize, kMSmem);
+  {
+    const cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_gemm_partials), kMSmem);
     if (e != cudaSuccess) return e;
-    configured = true;
   }
   if (K % kKB != 0 || splits < 1) return cudaErrorInvalidValue;
   CUtensorMap ta, tb;

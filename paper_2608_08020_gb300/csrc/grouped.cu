@@ -697,11 +697,9 @@ void make_kv_tensor_maps(gb_pool* pool) {
 
 template <int G>
 static cudaError_t launch_grouped_t(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(k_grouped<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+  {
+    const cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_grouped<G>), kSmem);
     if (e != cudaSuccess) return e;
-    configured = true;
   }
   const PoolView& v = pool->view;
   const float qscale = scale * 1.4426950408889634f;

@@ -300,6 +300,9 @@ inline void prof_end(gb_pool* p, int which, cudaStream_t s) {
   if (p->prof_stop[which]) prof_record(p->prof_stop[which], s);
 }
 gb_status check_launch(gb_pool* pool, const char* what);
+// Raise a kernel's dynamic shared memory limit to `bytes` on the current device.  The
+// attribute belongs to the device, so it is set once per (kernel, device), under a lock.
+cudaError_t set_max_dynamic_smem(const void* kernel, int bytes);
 
 
 // Kernel launchers implemented in the other translation units.

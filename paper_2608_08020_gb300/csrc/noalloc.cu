@@ -59,14 +59,21 @@ ScratchLayout scratch_layout(int beams, int Hkv, int W, int record_floats) {
 }
 
 // Work plan for caller-owned rows (one thread per row): every row with seq_len > 0 is
-// read whole.  Also clears the status word, the one scratch value that must start at zero.
+// read whole.  A row whose length is negative or longer than its table
+// (max_pages_per_beam x page_size tokens) is not read at all: its output is zero and the
+// call's status records GB_ERR_INVALID.  The status word, the one scratch value that must
+// start at zero, is cleared first.
 __global__ void __launch_bounds__(1024) k_noalloc_plan(PoolView v) {
   pdl_wait();
   pdl_launch_dependents();
   __shared__ int tmp[33];
   const int b = threadIdx.x;
+  if (b == 0) v.ctl[kCtlStatus] = GB_OK;
+  __syncthreads();
   const int L = b < v.max_beams ? v.seq_len[b] : 0;
-  const bool act = L > 0;
+  const bool bad = b < v.max_beams && (L < 0 || (long long)L > (long long)v.max_pages * v.P);
+  if (bad) set_status(v.ctl, GB_ERR_INVALID);
+  const bool act = L > 0 && !bad;
   const int n = act ? (L + kChunk - 1) / kChunk : 0;
   int total;
   const int off = block_exclusive_scan(n * v.Hkv, tmp, &total);
@@ -78,7 +85,6 @@ __global__ void __launch_bounds__(1024) k_noalloc_plan(PoolView v) {
   }
   if (b == 0) {
     plan_off(v, 0)[v.max_beams] = total;
-    v.ctl[kCtlStatus] = GB_OK;
     v.ctl[kCtlStepOk] = 1;
   }
 }
@@ -99,6 +105,9 @@ extern "C" gb_status gb_paged_decode_noalloc(const gb_paged_decode_args* a, gb_s
   const int G = a->num_q_heads / a->num_kv_heads;
   if (!decode_supported(a->kv_dtype, a->head_dim, G)) return GB_ERR_UNSUPPORTED;
   if (((uintptr_t)a->kv & 15) || ((uintptr_t)a->q & 15)) return GB_ERR_INVALID;
+  // The work plan counts 16-token chunks per (row, KV head) in 32-bit integers.
+  const long long max_chunks = ((long long)a->max_pages_per_beam * a->page_size + kChunk - 1) / kChunk;
+  if ((long long)a->num_beams * max_chunks * a->num_kv_heads >= (1ll << 31)) return GB_ERR_INVALID;
 
   int device = 0, sms = 0;
   if (cudaGetDevice(&device) != cudaSuccess || device < 0 || device >= kMaxDevices) return GB_ERR_CUDA;
@@ -138,5 +147,22 @@ extern "C" gb_status gb_paged_decode_noalloc(const gb_paged_decode_args* a, gb_s
   k_noalloc_plan<<<1, 1024, 0, s>>>(v);
   if (cudaGetLastError() != cudaSuccess) return GB_ERR_CUDA;
   if (launch_decode_view(v, W, 0, a->q, a->scale, a->out, s) != cudaSuccess) return GB_ERR_CUDA;
+  return GB_OK;
+}
+
+extern "C" gb_status gb_paged_decode_noalloc_status(int* device_status, gb_stream_t stream) {
+  if (!device_status) return GB_ERR_INVALID;
+  int device = 0;
+  if (cudaGetDevice(&device) != cudaSuccess || device < 0 || device >= kMaxDevices) return GB_ERR_CUDA;
+  void* base = nullptr;
+  if (scratch_address(device, &base) != cudaSuccess) return GB_ERR_CUDA;
+  // The status word is the first word of the scratch array (ScratchLayout::ctl = 0).
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int v = GB_OK;
+  if (cudaMemcpyAsync(&v, static_cast<const int*>(base) + kCtlStatus, sizeof(int), cudaMemcpyDeviceToHost, s) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(s) != cudaSuccess)
+    return GB_ERR_CUDA;
+  *device_status = v;
   return GB_OK;
 }

@@ -8,6 +8,9 @@
 // the order is exactly that sequential rule.
 #include <algorithm>
 #include <cstring>
+#include <mutex>
+#include <set>
+#include <tuple>
 #include <vector>
 
 #include "internal.cuh"
@@ -76,6 +79,19 @@ bool decode_supported(int dtype, int D, int G) {
 gb_status fail(gb_pool* pool, gb_status code, const char* what) {
   if (pool) pool->last_error = what;
   return code;
+}
+
+cudaError_t set_max_dynamic_smem(const void* kernel, int bytes) {
+  static std::mutex mu;
+  static std::set<std::tuple<const void*, int, int>> done;  // (kernel, device, bytes) already set
+  int device = 0;
+  cudaError_t e = cudaGetDevice(&device);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  if (done.count(std::make_tuple(kernel, device, bytes))) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done.insert(std::make_tuple(kernel, device, bytes));
+  return e;
 }
 
 gb_status check_launch(gb_pool* pool, const char* what) {
