@@ -45,18 +45,25 @@ if ROOT not in sys.path:
 def parse_args(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=0, help="timed decode steps (0: one tournament interval)")
+    ap.add_argument("--steps", type=int, default=0,
+                    help="timed decode steps (0: one tournament interval, or 64 where those inputs would not fit)")
     ap.add_argument("--warmup", type=int, default=8)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", type=int, default=2, help="workload index 1..5 (default 2: the metric's config)")
+    ap.add_argument("--config", type=int, default=5, choices=range(1, 7),
+                    help="workload index 1..6 (default 5: the 36-layer memory-capped step, the largest "
+                         "single-GPU workload; 6: independent roots with no shared KV)")
     ap.add_argument("--flags", choices=["auto", "per_beam"], default="auto")
     ap.add_argument("--group-min", type=int, default=0, help="beams a segment needs for the grouped path (0: library default, 2)")
-    ap.add_argument("--cpu-steps", type=int, default=200, help="steps of the oracle sample for cpu_baseline")
+    ap.add_argument("--cpu-steps", type=int, default=0,
+                    help="steps of the oracle sample for cpu_baseline (0: 200 layer-steps, i.e. 200 / layers)")
     ap.add_argument("--cpu-beams", type=int, default=16, help="beams per step in the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--beams", type=int, default=0, help="override the workload's beam count (smaller profiling cases)")
     ap.add_argument("--context", type=int, default=0, help="override the workload's context length")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="override the layer count, keeping the pool's page count (a one-layer copy of the "
+                         "36-layer workload has the same tree and the same per-layer kernels)")
     ap.add_argument("--probe", choices=["linear", "mlp", "seq"], default="linear",
                     help="scorer at the tournament points: the linear probe of the workloads, the two-layer MLP, "
                          "or the history-aware sequence scorer")
@@ -64,11 +71,10 @@ def parse_args(argv=None):
     ap.add_argument("--seq-shape", default="2,4,2,1024",
                     help="sequence scorer layers,q-heads,kv-heads,ffn (128-dim heads; d_model = q-heads x 128)")
     ap.add_argument("--breakdown", action="store_true",
-                    help="also time the planner, append and combine kernels (extra event records in the step)")
-    ap.add_argument("--event-stride", type=int, default=0,
-                    help="bracket the decode and grouped kernels with CUDA events on every n-th timed step "
-                         "(each event record splits the step's chain of dependent launches; 0: about 32 "
-                         "bracketed steps)")
+                    help="also time the planner, append and combine kernels in the profiled steps")
+    ap.add_argument("--profile-steps", type=int, default=16,
+                    help="steps before the timed window whose kernels the library brackets with CUDA events")
+    ap.add_argument("--no-capacity", action="store_true", help="skip the memory-capped workload's capacity search")
     ap.add_argument("--eager", action="store_true",
                     help="launch the timed steps one by one instead of as one captured CUDA graph")
     return ap.parse_args(argv)
@@ -83,10 +89,65 @@ def selected_workload(args, rank: int = 0):
         over["K"] = max(1, round(wl.K * args.beams / wl.beams))
     if args.context:
         over["context"] = args.context
+    if args.layers and args.layers != wl.num_layers:
+        over["num_layers"] = args.layers
+        over["num_pages"] = wl.pool_pages()       # the same page count, so the same tree
+        over["pool_bytes"] = None
     wl = dataclasses.replace(wl, **over)
-    if args.beams or args.context:
-        wl = dataclasses.replace(wl, name=f"{wl.name}[beams={wl.beams},context={wl.context}]")
+    if args.beams or args.context or args.layers:
+        wl = dataclasses.replace(wl, name=f"{wl.name}[beams={wl.beams},context={wl.context},layers={wl.num_layers}]")
     return wl
+
+
+INPUT_BUDGET_BYTES = 16 * 2**30  # device memory for the pre-generated step inputs
+
+
+def round_at(wl, L: int) -> bool:
+    """A probe + tournament round follows the decode step that brings the context to L."""
+    return L > wl.prompt_len and (L - wl.prompt_len) % wl.interval == 0
+
+
+def default_steps(wl, W: int, Kp: int, with_e2e: bool, step_input_bytes: int) -> int:
+    """Timed steps when --steps is 0: a tournament interval, at most 512 steps, 64 where the
+    pre-generated inputs of more would not fit beside the pool, and fewer where the phases
+    would not fit between the prompt and the context."""
+    K = min(wl.interval, 512)
+    if step_input_bytes * K > INPUT_BUDGET_BYTES:
+        K = 64
+    while K > 1:
+        try:
+            step_layout(wl, K, Kp, W, with_e2e)
+            return K
+        except SystemExit:
+            K //= 2
+    return K
+
+
+def step_layout(wl, K: int, Kp: int, W: int, with_e2e: bool) -> dict:
+    """Context lengths bounding each phase of the run, as (first, last) contexts of its steps
+    (a phase of n steps takes the context from first to first + n).  The timed window is the
+    last K steps: it ends at the workload's full context, where the schedule runs a probe +
+    tournament round, so the window holds every row of the hot path whatever K is.  Before it,
+    Kp profiled steps (kernels bracketed by events), and before those the K end-to-end steps,
+    which end at the last round boundary below the profiled steps when there is room (so they
+    hold a round too); untimed filler steps bridge the gap.  W warm-up steps come first."""
+    ctx, P0, delta = wl.context, wl.prompt_len, wl.interval
+    value = (ctx - K, ctx)
+    prof = (value[0] - Kp, value[0])
+    if with_e2e:
+        n = (prof[0] - P0) // delta
+        Re = P0 + n * delta if n >= 1 else None
+        if Re is None or Re - K - W < P0:
+            Re = prof[0]
+        e2e = (Re - K, Re)
+    else:
+        e2e = (prof[0], prof[0])
+    warm = (e2e[0] - W, e2e[0])
+    if warm[0] < P0:
+        raise SystemExit(f"{wl.name}: {W} warm-up + {K if with_e2e else 0} end-to-end + {Kp} profiled + {K} timed "
+                         f"steps do not fit between the prompt ({P0}) and the context ({ctx})")
+    return {"start": warm[0], "warmup": warm, "e2e": e2e, "filler": (e2e[1], prof[0]), "profile": prof,
+            "timed": value}
 
 
 # ---------------------------------------------------------------------------
@@ -150,19 +211,25 @@ def gpu_id_for_smi(local: int) -> str:
         return vis.split(",")[local] if vis else str(local)
 
 
-def captured_traffic(kernel: str, workload: str, path: str):
-    """DRAM bytes per launch from the committed ncu capture, if it is of this kernel source and workload."""
+def captured_traffic(kernel: str, workload: str, path: str, bytes_per_launch: float):
+    """DRAM bytes per launch from the committed ncu capture (profiles/traffic.json), if it is of this
+    kernel source, this workload and path, and a launch doing the same algorithmic work (within 3%);
+    None otherwise."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             rec = json.load(f).get(kernel)
         if not rec or rec["workload"] != workload or rec["path"] != path:
             return None
-        with open(os.path.join(ROOT, rec["source"]), "rb") as f:
-            if hashlib.sha256(f.read()).hexdigest() != rec["source_sha256"]:
-                return None
+        for src, sha in rec["sources"].items():
+            with open(os.path.join(ROOT, src), "rb") as f:
+                if hashlib.sha256(f.read()).hexdigest() != sha:
+                    return None
+        alg = rec["algorithmic_bytes_per_launch"]
+        if not bytes_per_launch or abs(alg - bytes_per_launch) > 0.03 * bytes_per_launch:
+            return None
         return rec["dram_bytes_per_launch"]
-    except (OSError, KeyError, ValueError):
+    except (OSError, KeyError, ValueError, TypeError):
         return None
 
 
@@ -271,7 +338,6 @@ def job_value(world: int, beams: int, steps: int, elapsed_ms: float) -> float:
 # ---------------------------------------------------------------------------
 # Our arm.
 # ---------------------------------------------------------------------------
-INPUT_BUDGET_BYTES = 16 * 2**30  # device memory for the pre-generated step inputs
 
 
 def capacity_search(wl, dev) -> dict:
@@ -363,13 +429,6 @@ class _Cudart:
         self._ok(self._wait(stream, e, 0), "cudaStreamWaitEvent")
 
 
-def bracketed_steps(W: int, K: int, event_stride: int, breakdown: bool):
-    """(stride, steps) of the timed steps whose kernels the library brackets with events:
-    every step under --breakdown, else every event_stride-th (0: about 32 of the K)."""
-    stride = 1 if breakdown else max(1, event_stride if event_stride > 0 else K // 32)
-    return stride, [i for i in range(W, W + K) if (i - W) % stride == 0]
-
-
 def build_seq_scorer(args, wl, g, dev, n_rounds_after: int):
     """The sequence scorer with seeded random weights and its step pool, seeded with the
     prompt's final hidden state and stepped once per tournament round already in the tree
@@ -403,7 +462,6 @@ def run_ours(args) -> None:
 
     from paper_2608_08020_gb300 import binding as B
     from workload import gen, gpu_gen
-    from workload.configs import BY_INDEX
     from workload.driver import GpuRun
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -419,47 +477,50 @@ def run_ours(args) -> None:
     C, Hq, Hkv, D, NL = wl.beams, wl.num_q_heads, wl.num_kv_heads, wl.head_dim, wl.num_layers
     esz_in = 2 if wl.kv_dtype == "bf16" else 4
     step_input_bytes = NL * C * (Hq + 2 * Hkv) * D * esz_in
-    if args.steps > 0:
-        K = args.steps
-    elif step_input_bytes * wl.interval > INPUT_BUDGET_BYTES:
-        K = 64                               # pre-generated inputs of a whole interval would not fit beside the pool
-    else:
-        K = wl.interval
-    S = W + (K if args.no_e2e else 2 * K)
+    Kp = max(1, args.profile_steps)
+    with_e2e = not args.no_e2e
+    K = args.steps if args.steps > 0 else default_steps(wl, W, Kp, with_e2e, step_input_bytes)
+    lay = step_layout(wl, K, Kp, W, with_e2e)
     delta = wl.interval
-    capacity = capacity_search(wl, dev) if (wl.pool_bytes is not None and rank == 0) else None
+    capacity = capacity_search(wl, dev) if (wl.pool_bytes is not None and rank == 0 and not args.no_capacity) else None
 
-    # A fixed pool holds the tree up to the workload's context: the steps end there.  Otherwise
-    # the timed window starts at the full context.
+    # Every phase ends at or before the workload's context, so the pool needs tables of that length.
     fixed_pool = wl.pool_bytes is not None
-    g = GpuRun(wl, device_gen=True, device=str(dev), max_context=wl.context + (0 if fixed_pool else S) + 1,
-               group_min_beams=args.group_min)
+    g = GpuRun(wl, device_gen=True, device=str(dev), max_context=wl.context + 1, group_min_beams=args.group_min)
     t_build = time.perf_counter()
-    g.build(upto=wl.context - (S if fixed_pool else W))  # the schedule's rounds up to here, then plain appends
+    g.build(upto=lay["start"])               # the schedule's rounds up to here, then plain appends
     torch.cuda.synchronize()
     t_build = time.perf_counter() - t_build
     pos0 = g.pos                             # context before the first (warm-up) step
+    assert pos0 == lay["start"]
+    S = wl.context - pos0                    # steps from here to the full context
 
-    def is_round(step: int) -> bool:         # a round follows the step that brings the context to L
-        L = pos0 + step + 1
-        return L > wl.prompt_len and (L - wl.prompt_len) % delta == 0
+    def is_round(i: int) -> bool:            # step i brings the context to pos0 + i + 1
+        return round_at(wl, pos0 + i + 1)
 
-    round_steps = [i for i in range(S) if is_round(i)]
-    # Step inputs for every step (and hidden states for the round steps), generated before timing.
-    qs = torch.empty(S, NL, C, Hq, D, dtype=g.tdt, device=dev)
-    ks = torch.empty(S, NL, C, Hkv, D, dtype=g.tdt, device=dev)
+    def steps_of(phase: str) -> range:
+        first, last = lay[phase]
+        return range(first - pos0, last - pos0)
+
+    # Step inputs (q, k, v of every layer) for K steps, generated on the device before any timing;
+    # every phase cycles through them (timing does not depend on their values).  The hidden states
+    # at each round are the seeded ones of that position, so the tree is the schedule's.
+    qs = torch.empty(K, NL, C, Hq, D, dtype=g.tdt, device=dev)
+    ks = torch.empty(K, NL, C, Hkv, D, dtype=g.tdt, device=dev)
     vs = torch.empty_like(ks)
-    hs = torch.empty(max(1, len(round_steps)), C, wl.hidden, dtype=g.hidden.dtype, device=dev)
-    h_index = {s: n for n, s in enumerate(round_steps)}
-    for i in range(S):
+    for j in range(K):
+        pos = lay["timed"][0] + j
         for l in range(NL):
-            gpu_gen.normal(qs[i, l], wl.kv_dtype, 1, C, Hq * D, [wl.seed, gen.TAG_Q, l, (0, 0, 1), pos0 + i],
+            gpu_gen.normal(qs[j, l], wl.kv_dtype, 1, C, Hq * D, [wl.seed, gen.TAG_Q, l, (0, 0, 1), pos],
                            scale=wl.q_scale if wl.q_scale is not None else 1.0)
             for which, dst in ((gen.TAG_KV_K, ks), (gen.TAG_KV_V, vs)):
-                gpu_gen.normal(dst[i, l], wl.kv_dtype, 1, C, Hkv * D, [wl.seed, which, l, (0, 0, 1), pos0 + i],
+                gpu_gen.normal(dst[j, l], wl.kv_dtype, 1, C, Hkv * D, [wl.seed, which, l, (0, 0, 1), pos],
                                row_scale=g.hscale_dev[l] if g.hscale else None, row_scale_div=D)
-    for s, n in h_index.items():
-        gpu_gen.normal(hs[n], wl.hidden_dtype, 1, C, wl.hidden, [wl.seed, gen.TAG_HIDDEN, (0, 0, 1), pos0 + s + 1])
+    round_steps = [i for i in range(S) if is_round(i)]
+    hs = torch.empty(max(1, len(round_steps)), C, wl.hidden, dtype=g.hidden.dtype, device=dev)
+    h_index = {s: n for n, s in enumerate(round_steps)}
+    for s_, n in h_index.items():
+        gpu_gen.normal(hs[n], wl.hidden_dtype, 1, C, wl.hidden, [wl.seed, gen.TAG_HIDDEN, (0, 0, 1), pos0 + s_ + 1])
     out = torch.empty(NL, C, Hq, D, dtype=torch.float32, device=dev)
     pool = g.pool
     mlp = None
@@ -475,6 +536,18 @@ def run_ours(args) -> None:
     if args.probe == "seq":       # the sequence scorer, seeded random weights, its own step pool
         seq = build_seq_scorer(args, wl, g, dev, n_rounds_after=len(round_steps))
     stream = torch.cuda.current_stream()
+    PROF = (B.GB_PROF_DECODE, B.GB_PROF_PROBE, B.GB_PROF_PRUNE, B.GB_PROF_GROUPED, B.GB_PROF_PLAN,
+            B.GB_PROF_APPEND, B.GB_PROF_COMBINE, B.GB_PROF_ATTENTION)
+
+    def clear_prof():
+        for which in PROF:
+            B.gb_pool_set_profile_events(pool.handle, which, None, None)
+            if seq is not None:
+                B.gb_pool_set_profile_events(seq.pool.handle, which, None, None)
+
+    def inputs(i):
+        j = i % K
+        return qs[j], ks[j], vs[j], hs[h_index.get(i, 0)]
 
     def step(i, q, k, v, h, prof=None, o=None):
         o = out if o is None else o
@@ -489,12 +562,14 @@ def run_ours(args) -> None:
                     if l == 0:
                         B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PLAN, *prof["plan"])
             pool.decode_attention(l, q[l], k[l], v[l], wl.attn_scale, o[l], flags)
+        if prof is not None:
+            clear_prof()
         if is_round(i):
-            if prof is not None:
+            if prof is not None and "probe" in prof:
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PROBE, *prof["probe"])
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_PRUNE, *prof["prune"])
             if seq is not None:
-                if prof is not None:
+                if prof is not None and "probe" in prof:
                     B.gb_pool_set_profile_events(seq.pool.handle, B.GB_PROF_PROBE, *prof["probe"])
                     B.gb_pool_set_profile_events(seq.pool.handle, B.GB_PROF_PRUNE, *prof["fork"])
                 seq.step(h, g.scores)
@@ -506,177 +581,36 @@ def run_ours(args) -> None:
             pool.prune_branch(wl.K, wl.fanout, wl.warmup, None, g.parent, g.pruned, g.lineage)
             if seq is not None:
                 seq.fork(g.parent)
+            if prof is not None:
+                clear_prof()
 
-    for i in range(W):
-        step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)])
-    torch.cuda.synchronize()
-
-    # Per-kernel events, recorded by the library on this stream around the kernels.
     def ev_pair():
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         b.record(stream)
         return a, b
-    timed_rounds = [i for i in range(W, W + K) if is_round(i)]
-    stride, inst = bracketed_steps(W, K, args.event_stride, args.breakdown)
-    profs = {i: {} for i in range(W, W + K)}
-    for i in inst:
-        profs[i].update({"dec": [ev_pair() for _ in range(NL)], "gr": [ev_pair() for _ in range(NL)],
-                         "att": [ev_pair() for _ in range(NL)]})
-    if args.breakdown:  # every kernel of the step bracketed (the extra event records cost step time)
-        for i in inst:
-            profs[i].update({"app": [ev_pair() for _ in range(NL)], "comb": [ev_pair() for _ in range(NL)],
-                             "plan": ev_pair()})
-    for i in timed_rounds:
-        profs[i]["probe"], profs[i]["prune"], profs[i]["fork"] = ev_pair(), ev_pair(), ev_pair()
-    torch.cuda.synchronize()
-    launches0 = B.gb_pool_launch_count(pool.handle)
-    seq_launches0 = B.gb_pool_launch_count(seq.pool.handle) if seq is not None else 0
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    graph = None
-    if not args.eager:
-        # The K timed steps are captured once into a CUDA graph and launched once, so the
-        # host's per-launch cost is out of the step (every kernel still runs, once, with the
-        # arguments of its own step; the library's event records become graph nodes).
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph):
-            for i in range(W, W + K):
-                step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)], profs[i])
-        torch.cuda.synchronize()
-    clocks = ClockSampler(gpu_id_for_smi(local))
-    clocks.start()
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    t_start.record(stream)
-    torch.cuda.nvtx.range_push("timed")  # lets a profiler capture exactly the timed steps
-    if graph is not None:
-        graph.replay()
-    else:
-        for i in range(W, W + K):
-            step(i, qs[i], ks[i], vs[i], hs[h_index.get(i, 0)], profs[i])
-    torch.cuda.nvtx.range_pop()
-    t_end.record(stream)
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    clk = clocks.stop()
-    for which in (B.GB_PROF_DECODE, B.GB_PROF_PROBE, B.GB_PROF_PRUNE, B.GB_PROF_GROUPED, B.GB_PROF_PLAN,
-                  B.GB_PROF_APPEND, B.GB_PROF_COMBINE, B.GB_PROF_ATTENTION):
-        B.gb_pool_set_profile_events(pool.handle, which, None, None)
-        if seq is not None:
-            B.gb_pool_set_profile_events(seq.pool.handle, which, None, None)
-    stats = B.gb_pool_read_step_stats(pool.handle, max_steps=K)  # one record per timed step
-    launches = B.gb_pool_launch_count(pool.handle) - launches0
-    if seq is not None:
-        launches += B.gb_pool_launch_count(seq.pool.handle) - seq_launches0
-        if seq.pool.status() != 0:
-            raise RuntimeError("sequence scorer's step pool reported an error: the measurement is invalid")
-    elapsed_ms = max_over_ranks(t_start.elapsed_time(t_end), world, dev)
-    status = pool.status()
-    if status != 0:
-        raise RuntimeError(f"device status {status} after the timed steps: the measurement is invalid")
-    dec_ms = [a.elapsed_time(b) for i in inst for a, b in profs[i]["dec"]]
-    gr_ms = [a.elapsed_time(b) for i in inst for a, b in profs[i]["gr"]]
-    att_ms = [a.elapsed_time(b) for i in inst for a, b in profs[i]["att"]]
-    # In-stream duration of every kernel of a decode step (per layer; the planner once per step).
-    step_kernels_us = None
-    if args.breakdown:
-        step_kernels_us = {
-            "plan": statistics.mean(profs[i]["plan"][0].elapsed_time(profs[i]["plan"][1]) for i in inst) * 1e3,
-            "append": statistics.mean(a.elapsed_time(b) for i in inst for a, b in profs[i]["app"]) * 1e3,
-            "grouped": statistics.mean(gr_ms) * 1e3,
-            "decode": statistics.mean(dec_ms) * 1e3,
-            "combine": statistics.mean(a.elapsed_time(b) for i in inst for a, b in profs[i]["comb"]) * 1e3,
-        }
-    prune_us = statistics.mean(profs[i]["prune"][0].elapsed_time(profs[i]["prune"][1]) for i in timed_rounds) * 1e3 \
-        if timed_rounds else None
-    probe_us = statistics.mean(profs[i]["probe"][0].elapsed_time(profs[i]["probe"][1]) for i in timed_rounds) * 1e3 \
-        if timed_rounds else None
-    fork_us = statistics.mean(profs[i]["fork"][0].elapsed_time(profs[i]["fork"][1]) for i in timed_rounds) * 1e3 \
-        if (timed_rounds and seq is not None) else None
-    grouped_on = flags != B.GB_PATH_PER_BEAM and wl.kv_dtype == "bf16" and D == 128
-    # The per-beam kernel: warp-level MMAs for bf16 pools with 128-dim heads, paired fp32 FMAs otherwise.
-    dec = "k_decode_mma" if wl.kv_dtype == "bf16" and D == 128 else "k_decode"
 
-    # Algorithmic work per launch, from the library's per-step records:
-    #   per-beam:  tokens it reads (all KV heads, K and V) + the queries;
-    #   k_grouped: K/V tiles it reads (once per 128-row query tile) and the useful flops
-    #              4 * D per (query row, token) for Q.K^T and P.V.
-    esz = 2 if wl.kv_dtype == "bf16" else 4
-    kv_tok = 2 * Hkv * D * esz
-    q_bytes = C * Hq * D * esz
-    assert len(stats) == K, (len(stats), K)
-    stats = [stats[i - W] for i in inst]       # the bracketed steps' work, to match their durations
-    dec_tokens = [int(s[1] if grouped_on else s[0]) for s in stats]
-    dec_bytes = statistics.mean(t * kv_tok + q_bytes for t in dec_tokens)
-    eff_bytes = statistics.mean(int(s[0]) * kv_tok + q_bytes for s in stats)   # as if every beam read everything
-    gr_bytes = statistics.mean(Hkv * int(s[3]) * 2 * D * esz for s in stats) if grouped_on else 0.0
-    gr_flops = statistics.mean(Hkv * int(s[2]) * 4 * D for s in stats) if grouped_on else 0.0
-    dec_avg_s = statistics.mean(dec_ms) / 1e3
-    gr_avg_s = statistics.mean(gr_ms) / 1e3 if grouped_on else 0.0
-    achieved = dec_bytes / dec_avg_s / 1e9
-    peaks = measured_peaks()
-    peak = peaks.get("hbm_gbs")
-    peak_src = "measured" if peak else "fallback"
-    peak = peak or 6800.0
-    tpeak = peaks.get("bf16_tflops_sustained") or peaks.get("bf16_tflops")
-    tpeak_src = "measured sustained" if tpeak else "fallback"
-    tpeak = tpeak or 1700.0
-    kernels = {dec: {"us": dec_avg_s * 1e6, "bytes": dec_bytes, "gbps": achieved, "frac_hbm": achieved / peak}}
-    if grouped_on and gr_avg_s > 0:
-        kernels["k_grouped"] = {"us": gr_avg_s * 1e6, "bytes": gr_bytes, "gbps": gr_bytes / gr_avg_s / 1e9,
-                                "frac_hbm": gr_bytes / gr_avg_s / 1e9 / peak, "flops": gr_flops,
-                                "tflops": gr_flops / gr_avg_s / 1e12, "frac_tensor": gr_flops / gr_avg_s / 1e12 / tpeak,
-                                "segments": statistics.mean(int(s[4]) for s in stats),
-                                "work_units": statistics.mean(int(s[5]) * Hkv for s in stats)}
-    att_avg_s = statistics.mean(att_ms) / 1e3
-    dominant = "k_grouped" if "k_grouped" in kernels and gr_avg_s > dec_avg_s else dec
-    if "k_grouped" in kernels:
-        # The grouped and per-beam kernels run concurrently on disjoint SMs: the pair is
-        # one phase of the step, timed from before the fork to after the join.
-        tr = [captured_traffic(k, wl.name, args.flags) for k in ("k_grouped", dec)]
-        pair_bytes = gr_bytes + dec_bytes
-        roofline = {"bound": "hbm", "kernel": f"k_grouped + {dec} (concurrent, disjoint SMs)",
-                    "achieved": pair_bytes / att_avg_s / 1e9, "peak": peak, "unit": "GB/s",
-                    "frac": pair_bytes / att_avg_s / 1e9 / peak,
-                    "traffic": (tr[0] + tr[1]) if None not in tr else None, "bytes_per_launch": pair_bytes,
-                    "phase_us": att_avg_s * 1e6, "peak_source": f"{peak_src} hbm_gbs"}
-    elif dominant == dec:
-        roofline = {"bound": "hbm", "kernel": f"{dec} (split-KV decode)", "achieved": achieved, "peak": peak,
-                    "unit": "GB/s", "frac": achieved / peak, "traffic": captured_traffic(dec, wl.name, args.flags), "bytes_per_launch": dec_bytes,
-                    "peak_source": f"{peak_src} hbm_gbs"}
-    else:
-        kg = kernels["k_grouped"]
-        if kg["frac_tensor"] >= kg["frac_hbm"]:
-            roofline = {"bound": "tensor", "kernel": "k_grouped (tcgen05 shared-prefix)", "achieved": kg["tflops"],
-                        "peak": tpeak, "unit": "TFLOP/s", "frac": kg["frac_tensor"], "traffic": captured_traffic("k_grouped", wl.name, args.flags),
-                        "flops_per_launch": gr_flops, "peak_source": f"{tpeak_src} bf16_tflops"}
-        else:
-            roofline = {"bound": "hbm", "kernel": "k_grouped (tcgen05 shared-prefix)", "achieved": kg["gbps"],
-                        "peak": peak, "unit": "GB/s", "frac": kg["frac_hbm"], "traffic": captured_traffic("k_grouped", wl.name, args.flags),
-                        "bytes_per_launch": gr_bytes, "peak_source": f"{peak_src} hbm_gbs"}
+    # ---- warm-up --------------------------------------------------------------------------
+    for i in steps_of("warmup"):
+        step(i, *inputs(i))
+    torch.cuda.synchronize()
 
-    value = job_value(world, C, K, elapsed_ms)
-    ms_per_step = elapsed_ms / K
-
-    # End to end through the C ABI with host buffers: each step's inputs copied in from pinned
-    # memory and its outputs read back, inside the timed region.
+    # ---- end to end through the C ABI with host buffers ----------------------------------------
+    # Every step's q, k, v (and, at a round, the hidden states) come from pinned host memory in
+    # one copy, and the step's attention output (and, at a round, the scores and the tournament's
+    # outputs) go back to pinned host memory, inside the timed region.  Copies run on a second
+    # stream into double buffers, overlapping the previous step.
     e2e = None
-    if not args.no_e2e:
-        # End to end: every step's q, k, v (and, at a round, the hidden states) come from
-        # pinned host memory in one copy, and the step's attention output (and, at a round,
-        # the scores and the tournament's outputs) go back to pinned host memory.  Copies
-        # run on a second stream into double buffers, overlapping the previous step.
-        sl = range(W + K, W + 2 * K)
+    sl = steps_of("e2e")
+    if with_e2e:
         parts = (qs, ks, vs)
         nbytes = [t[0].numel() * t.element_size() for t in parts]
         offs = [0, nbytes[0], nbytes[0] + nbytes[1]]
         in_bytes = sum(nbytes)
         hin = torch.empty((K, in_bytes), dtype=torch.uint8).pin_memory()
-        for n, i in enumerate(sl):
+        for n in range(K):
             for t, o0, nb in zip(parts, offs, nbytes):
-                hin[n, o0:o0 + nb].copy_(t[i].reshape(-1).view(torch.uint8).cpu())
+                hin[n, o0:o0 + nb].copy_(t[n].reshape(-1).view(torch.uint8).cpu())
         hh = hs.cpu().pin_memory()
         din = [torch.empty(in_bytes, dtype=torch.uint8, device=dev) for _ in range(2)]
         views = [[din[b][o0:o0 + nb].view(t.dtype).view(t[0].shape) for t, o0, nb in zip(parts, offs, nbytes)]
@@ -688,7 +622,7 @@ def run_ours(args) -> None:
                for n, i in enumerate(sl) if is_round(i)}
         cs = torch.cuda.Stream(device=dev)
         rt = _Cudart()
-        S, CS = stream.cuda_stream, cs.cuda_stream
+        SS, CS = stream.cuda_stream, cs.cuda_stream
         loaded, done, outfree = ([rt.event() for _ in range(2)] for _ in range(3))
         ev_fork, ev_join = rt.event(), rt.event()
         out_bytes = dout[0].numel() * dout[0].element_size()
@@ -706,7 +640,7 @@ def run_ours(args) -> None:
             b = n % 2
             if n >= 2:
                 rt.wait(CS, done[b])
-            rt.copy(din[b].data_ptr(), hin[n].data_ptr(), in_bytes, rt.H2D, CS)
+            rt.copy(din[b].data_ptr(), hin[n % K].data_ptr(), in_bytes, rt.H2D, CS)
             h2d += in_bytes
             if is_round(sl[n]):
                 nb = hh[0].numel() * hh.element_size()
@@ -716,23 +650,23 @@ def run_ours(args) -> None:
 
         e0.record(stream)
         t_host = time.perf_counter()
-        rt.record(ev_fork, S)
+        rt.record(ev_fork, SS)
         rt.wait(CS, ev_fork)
         load(0)
         for n, i in enumerate(sl):
             b = n % 2
-            if n + 1 < K:
+            if n + 1 < len(sl):
                 load(n + 1)
-            rt.wait(S, loaded[b])
+            rt.wait(SS, loaded[b])
             if n >= 2:
-                rt.wait(S, outfree[b])
+                rt.wait(SS, outfree[b])
             if is_round(i):
                 step(i, *views[b], h_d[b], o=dout[b])
             else:
                 for l in range(NL):
                     qp, kp, vp, op = ptrs[b][l]
-                    B.gb_decode_attention(pool.handle, l, qp, kp, vp, wl.attn_scale, op, flags, S)
-            rt.record(done[b], S)
+                    B.gb_decode_attention(pool.handle, l, qp, kp, vp, wl.attn_scale, op, flags, SS)
+            rt.record(done[b], SS)
             rt.wait(CS, done[b])
             rt.copy(o_h[b].data_ptr(), dout[b].data_ptr(), out_bytes, rt.D2H, CS)
             d2h += out_bytes
@@ -743,27 +677,182 @@ def run_ours(args) -> None:
                     d2h += nb
             rt.record(outfree[b], CS)
         rt.record(ev_join, CS)
-        rt.wait(S, ev_join)
+        rt.wait(SS, ev_join)
         e1.record(stream)
         t_host = time.perf_counter() - t_host
         torch.cuda.synchronize()
         for e in loaded + done + outfree + [ev_fork, ev_join]:
             rt.destroy(e)
         e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
-        e2e = {"value": job_value(world, C, K, e_ms), "unit": "beam-tokens/s", "h2d_bytes_per_step": int(h2d // K),
-               "d2h_bytes_per_step": int(d2h // K), "ms_per_step": e_ms / K,
-               "host_issue_us_per_step": t_host / K * 1e6,
-               "path": "eager calls of the C API (gb_decode_attention per layer and step); inputs copied from "
-                       "pinned host memory and outputs read back every step with cudaMemcpyAsync, on a copy "
-                       "stream double-buffered against compute"}
+        e2e_rounds = sum(1 for i in sl if is_round(i))
+        e2e = {"value": job_value(world, C, len(sl), e_ms), "unit": "beam-tokens/s", "h2d_bytes_per_step": int(h2d // len(sl)),
+               "d2h_bytes_per_step": int(d2h // len(sl)), "ms_per_step": e_ms / len(sl),
+               "host_issue_us_per_step": t_host / len(sl) * 1e6,
+               "context": [lay["e2e"][0], lay["e2e"][1]], "rounds": e2e_rounds,
+               "path": "eager calls of the C API (gb_decode_attention per layer and step; probe and tournament "
+                       "at a round); inputs copied from pinned host memory and outputs read back every step with "
+                       "cudaMemcpyAsync, on a copy stream double-buffered against compute"}
         status = pool.status()
         if status != 0:
             raise RuntimeError(f"device status {status} after the e2e steps: the measurement is invalid")
+        del hin, hh, din, views, dout, o_h
+
+    # ---- filler: untimed steps up to the profiled steps ---------------------------------------
+    for i in steps_of("filler"):
+        step(i, *inputs(i))
+    torch.cuda.synchronize()
+
+    # ---- profiled steps: every kernel of the step bracketed by events ---------------------------
+    # Each event record splits the step's chain of programmatically dependent launches, so the
+    # kernel durations come from these steps and the timed window below carries no such records.
+    pl = list(steps_of("profile"))
+    profs = {i: {"dec": [ev_pair() for _ in range(NL)], "gr": [ev_pair() for _ in range(NL)],
+                 "att": [ev_pair() for _ in range(NL)]} for i in pl}
+    if args.breakdown:
+        for i in pl:
+            profs[i].update({"app": [ev_pair() for _ in range(NL)], "comb": [ev_pair() for _ in range(NL)],
+                             "plan": ev_pair()})
+    torch.cuda.synchronize()
+    if args.eager:
+        for i in pl:
+            step(i, *inputs(i), prof=profs[i])
+    else:
+        pgraph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(pgraph):
+            for i in pl:
+                step(i, *inputs(i), prof=profs[i])
+        pgraph.replay()
+    torch.cuda.synchronize()
+    stats = B.gb_pool_read_step_stats(pool.handle, max_steps=len(pl))   # one record per profiled step
+    assert len(stats) == len(pl), (len(stats), len(pl))
+    dec_ms = [a.elapsed_time(b) for i in pl for a, b in profs[i]["dec"]]
+    gr_ms = [a.elapsed_time(b) for i in pl for a, b in profs[i]["gr"]]
+    att_ms = [a.elapsed_time(b) for i in pl for a, b in profs[i]["att"]]
+    step_kernels_us = None
+    if args.breakdown:
+        step_kernels_us = {
+            "plan": statistics.mean(profs[i]["plan"][0].elapsed_time(profs[i]["plan"][1]) for i in pl) * 1e3,
+            "append": statistics.mean(a.elapsed_time(b) for i in pl for a, b in profs[i]["app"]) * 1e3,
+            "grouped": statistics.mean(gr_ms) * 1e3,
+            "decode": statistics.mean(dec_ms) * 1e3,
+            "combine": statistics.mean(a.elapsed_time(b) for i in pl for a, b in profs[i]["comb"]) * 1e3,
+        }
+
+    # ---- the timed window: K steps ending at the full context, then that context's round ---------
+    tl = list(steps_of("timed"))
+    timed_rounds = [i for i in tl if is_round(i)]
+    rprof = {i: {} for i in tl}
+    for i in timed_rounds:      # the round's probe and tournament (after the window's last decode step)
+        rprof[i] = {"probe": ev_pair(), "prune": ev_pair(), "fork": ev_pair()}
+    torch.cuda.synchronize()
+    launches0 = B.gb_pool_launch_count(pool.handle)
+    seq_launches0 = B.gb_pool_launch_count(seq.pool.handle) if seq is not None else 0
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    graph = None
+    if not args.eager:
+        # The K timed steps are captured once into a CUDA graph and launched once, so the
+        # host's per-launch cost is out of the step (every kernel still runs, once, with the
+        # arguments of its own step).
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            for i in tl:
+                step(i, *inputs(i), prof=rprof[i] or None)
+        torch.cuda.synchronize()
+    clocks = ClockSampler(gpu_id_for_smi(local))
+    clocks.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    torch.cuda.nvtx.range_push("timed")  # lets a profiler capture exactly the timed steps
+    if graph is not None:
+        graph.replay()
+    else:
+        for i in tl:
+            step(i, *inputs(i), prof=rprof[i] or None)
+    torch.cuda.nvtx.range_pop()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    clear_prof()
+    launches = B.gb_pool_launch_count(pool.handle) - launches0
+    if seq is not None:
+        launches += B.gb_pool_launch_count(seq.pool.handle) - seq_launches0
+        if seq.pool.status() != 0:
+            raise RuntimeError("sequence scorer's step pool reported an error: the measurement is invalid")
+    elapsed_ms = max_over_ranks(t_start.elapsed_time(t_end), world, dev)
+    status = pool.status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after the timed steps: the measurement is invalid")
+    prune_us = statistics.mean(rprof[i]["prune"][0].elapsed_time(rprof[i]["prune"][1]) for i in timed_rounds) * 1e3 \
+        if timed_rounds else None
+    probe_us = statistics.mean(rprof[i]["probe"][0].elapsed_time(rprof[i]["probe"][1]) for i in timed_rounds) * 1e3 \
+        if timed_rounds else None
+    fork_us = statistics.mean(rprof[i]["fork"][0].elapsed_time(rprof[i]["fork"][1]) for i in timed_rounds) * 1e3 \
+        if (timed_rounds and seq is not None) else None
+    grouped_on = flags != B.GB_PATH_PER_BEAM and wl.kv_dtype == "bf16" and D == 128
+    # The per-beam kernel: warp-level MMAs for bf16 pools with 128-dim heads, paired fp32 FMAs otherwise.
+    dec = "k_decode_mma" if wl.kv_dtype == "bf16" and D == 128 else "k_decode"
+
+    # Algorithmic work per launch, from the library's per-step records of the profiled steps:
+    #   per-beam kernel: the tokens it reads (all KV heads, K and V) + the queries;
+    #   k_grouped: unique bytes = every shared segment's pages once (K and V of every KV head);
+    #              bytes_read = the K/V tiles it reads (once per 128-row query tile);
+    #              useful flops = 4 * D per (query row, token) for Q.K^T and P.V.
+    esz = 2 if wl.kv_dtype == "bf16" else 4
+    kv_tok = 2 * Hkv * D * esz
+    q_bytes = C * Hq * D * esz
+    dec_tokens = [int(s[1] if grouped_on else s[0]) for s in stats]
+    dec_bytes = statistics.mean(t * kv_tok + q_bytes for t in dec_tokens)
+    eff_bytes = statistics.mean(int(s[0]) * kv_tok + q_bytes for s in stats)   # as if every beam read everything
+    gr_read = statistics.mean(Hkv * int(s[3]) * 2 * D * esz for s in stats) if grouped_on else 0.0
+    gr_unique = statistics.mean(int(s[8]) * kv_tok for s in stats) if grouped_on else 0.0
+    gr_flops = statistics.mean(Hkv * int(s[2]) * 4 * D for s in stats) if grouped_on else 0.0
+    dec_avg_s = statistics.mean(dec_ms) / 1e3
+    gr_avg_s = statistics.mean(gr_ms) / 1e3 if grouped_on else 0.0
+    achieved = dec_bytes / dec_avg_s / 1e9
+    peaks = measured_peaks()
+    peak = peaks.get("hbm_gbs")
+    peak_src = "measured" if peak else "fallback"
+    peak = peak or 6800.0
+    tpeak = peaks.get("bf16_tflops_sustained") or peaks.get("bf16_tflops")
+    tpeak_src = "measured sustained" if tpeak else "fallback"
+    tpeak = tpeak or 1700.0
+    kernels = {dec: {"us": dec_avg_s * 1e6, "bytes": dec_bytes, "gbps": achieved, "frac_hbm": achieved / peak}}
+    if grouped_on and gr_avg_s > 0:
+        kernels["k_grouped"] = {"us": gr_avg_s * 1e6, "bytes": gr_unique, "bytes_read": gr_read,
+                                "gbps": gr_unique / gr_avg_s / 1e9, "frac_hbm": gr_unique / gr_avg_s / 1e9 / peak,
+                                "gbps_read": gr_read / gr_avg_s / 1e9, "flops": gr_flops,
+                                "tflops": gr_flops / gr_avg_s / 1e12, "frac_tensor": gr_flops / gr_avg_s / 1e12 / tpeak,
+                                "segments": statistics.mean(int(s[4]) for s in stats),
+                                "work_units": statistics.mean(int(s[5]) * Hkv for s in stats)}
+    att_avg_s = statistics.mean(att_ms) / 1e3
+    if "k_grouped" in kernels:
+        # The grouped and per-beam kernels form one phase of the step (they run side by side, or
+        # back to back on two streams), timed from before the fork to after the join.
+        pair_bytes = gr_unique + dec_bytes
+        tr = captured_traffic("k_grouped+" + dec, wl.name, args.flags, pair_bytes)
+        roofline = {"bound": "hbm", "kernel": f"k_grouped + {dec} (the attention phase)",
+                    "achieved": pair_bytes / att_avg_s / 1e9, "peak": peak, "unit": "GB/s",
+                    "frac": pair_bytes / att_avg_s / 1e9 / peak, "traffic": tr, "bytes_per_launch": pair_bytes,
+                    "bytes_read_per_launch": gr_read + dec_bytes, "phase_us": att_avg_s * 1e6,
+                    "peak_source": f"{peak_src} hbm_gbs"}
+    else:
+        roofline = {"bound": "hbm", "kernel": f"{dec} (split-KV decode)", "achieved": achieved, "peak": peak,
+                    "unit": "GB/s", "frac": achieved / peak,
+                    "traffic": captured_traffic(dec, wl.name, args.flags, dec_bytes), "bytes_per_launch": dec_bytes,
+                    "peak_source": f"{peak_src} hbm_gbs"}
+
+    value = job_value(world, C, K, elapsed_ms)
+    ms_per_step = elapsed_ms / K
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = oracle_sample(wl, args.cpu_steps, args.cpu_beams)
-        one = oracle_sample(wl, max(1, args.cpu_steps // 8), 2, workers=1)   # the same oracle on one core
+        cpu_steps = args.cpu_steps or max(2, 200 // NL)
+        cpu = oracle_sample(wl, cpu_steps, args.cpu_beams)
+        one = oracle_sample(wl, max(1, cpu_steps // 8), 2, workers=1)   # the same oracle on one core
         cpu["single_core"] = {"value": one["value"], "unit": one["unit"], "seconds": one["seconds"],
                               "sample": one["sample"]}
     if rank == 0:
@@ -772,23 +861,24 @@ def run_ours(args) -> None:
             "value": value, "unit": "beam-tokens/s", "n_gpus": world, "steps": K, "warmup": W,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": wl.kv_dtype, "data": "synthetic (seeded counter-based generator, generated on device)",
-            "config": {"workload": wl.name, "beams": C, "context_at_start": pos0 + W, "context_at_end": pos0 + W + K,
-                       "layers": NL, "heads": f"{Hq}/{Hkv}", "head_dim": D, "page_size": wl.page_size,
-                       "kv_dtype": wl.kv_dtype,
+            "config": {"workload": wl.name, "beams": C, "context_at_start": lay["timed"][0],
+                       "context_at_end": lay["timed"][1], "layers": NL, "heads": f"{Hq}/{Hkv}", "head_dim": D,
+                       "page_size": wl.page_size, "kv_dtype": wl.kv_dtype,
                        "schedule": f"decode every step; probe + tournament (K={wl.K}, fanout {wl.fanout}) every "
-                                   f"{delta} tokens: {len(timed_rounds)} round(s) in the timed window",
+                                   f"{delta} tokens: {len(timed_rounds)} round(s) in the timed window (at its end)",
                        "path": args.flags, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "launch": "eager" if args.eager else "one CUDA graph of the timed steps",
-                       "kernel_events": f"decode and grouped kernels bracketed by CUDA events on {len(inst)} of the "
-                                        f"{K} timed steps (every {stride})",
+                       "kernel_events": f"none in the timed window but the round's probe and tournament; kernel "
+                                        f"durations from {len(pl)} profiled steps just before it "
+                                        f"(contexts {lay['profile'][0]}-{lay['profile'][1]})",
                        "probe": {"linear": "linear", "mlp": f"mlp (hidden {args.mlp_hidden})",
                                  "seq": f"sequence scorer (layers, q heads, kv heads, ffn = {args.seq_shape}; "
                                         f"step pool of {seq.history} positions per trace before the window)"
                                  if seq is not None else None}[args.probe],
-                       "l2": f"inputs larger than L2: {eff_bytes / 2**30:.2f} GiB of per-beam KV reads per step",
+                       "l2": f"inputs larger than L2: {eff_bytes / 2**30:.2f} GiB of per-beam KV reads per layer-step",
                        "tree_build_s": round(t_build, 2),
-                       "window": (f"steps end at the full context {wl.context} (fixed {wl.pool_bytes / 1e9:.0f} GB pool)"
-                                  if fixed_pool else f"steps start at the full context {wl.context}")},
+                       "window": (f"steps end at the full context {wl.context} (fixed {wl.pool_bytes / 1e9:.0f} GB "
+                                  f"pool)" if fixed_pool else f"steps end at the full context {wl.context}")},
             "attention_us": att_avg_s * 1e6,
             "attention_tbps": eff_bytes / att_avg_s / 1e12,
             "attention_tbps_note": "every beam's whole context (K and V of all KV heads) per attention time",
@@ -797,6 +887,8 @@ def run_ours(args) -> None:
             "step_kernels_us": step_kernels_us,
             "probe_us": probe_us,
             "prune_branch_us": prune_us,
+            "prune_branch_note": "the whole gb_prune_branch call: rank, route, fork tables, refcounts, free, "
+                                 "and the shared-prefix segment rebuild",
             "scorer_fork_us": fork_us,
             "kernels": kernels,
             "capacity": capacity,
@@ -820,18 +912,22 @@ def run_reference(args) -> None:
     wl = selected_workload(args)
     W = args.warmup
     K = args.steps if args.steps > 0 else wl.interval
-    # Each step: a bounded sample (a few beams) so W + K steps end within minutes.
+    # Each step: a bounded sample (a few beams, every layer) so that the run ends within minutes:
+    # at most 400 layer-steps per worker process.
     per_step_beams = max(1, min(args.cpu_beams, 16))
-    res = oracle_sample(wl, W + K, per_step_beams)
-    steps_total = W + K
+    steps_total = max(1, min(W + K, 400 // wl.num_layers))
+    res = oracle_sample(wl, steps_total, per_step_beams)
     line = {
         "impl": "reference",
         "metric": "beam-decode attn beam-tokens/s + achieved HBM TB/s vs peak; prune+branch us/step",
         "value": res["value"], "unit": "beam-tokens/s", "n_gpus": int(os.environ.get("WORLD_SIZE", "1")),
-        "steps": K, "warmup": W, "ms_per_step": res["seconds"] * 1e3 / steps_total, "higher_is_better": True,
+        "steps": K, "warmup": W, "ms_per_step": wl.beams / res["value"] * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded counter-based generator)",
-        "config": {"workload": wl.name, "beams": wl.beams, "context": wl.context},
+        "config": {"workload": wl.name, "beams": wl.beams, "context": wl.context, "layers": wl.num_layers,
+                   "heads": f"{wl.num_q_heads}/{wl.num_kv_heads}", "head_dim": wl.head_dim,
+                   "page_size": wl.page_size, "kv_dtype": wl.kv_dtype,
+                   "sample_steps": steps_total, "sample_beams_per_step": per_step_beams},
         "cpu_baseline": {"value": res["value"], "unit": res["unit"], "cores": res["cores"], "kind": "oracle",
                          "sample": res["sample"]},
         "e2e": {"value": res["value"], "unit": "beam-tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

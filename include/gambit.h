@@ -263,7 +263,8 @@ gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_strea
  * following calls on this pool, so a caller can time that kernel alone on its
  * own stream: `which` is GB_PROF_DECODE (the split-KV decode kernel of
  * gb_decode_attention), GB_PROF_PROBE (gb_score_probe, gb_score_mlp, or all of
- * gb_scorer_step), GB_PROF_PRUNE (gb_prune_branch or gb_fork_slots), GB_PROF_GROUPED (the grouped shared-prefix kernel),
+ * gb_scorer_step), GB_PROF_PRUNE (all of gb_prune_branch or gb_fork_slots, the
+ * shared-prefix segment rebuild included), GB_PROF_GROUPED (the grouped shared-prefix kernel),
  * GB_PROF_PLAN (the step planner: page allocation and decode plans, layer 0),
  * GB_PROF_APPEND (the K/V append of a layer), GB_PROF_COMBINE (the merge of
  * partial results) or GB_PROF_ATTENTION (the attention kernels of a layer: the grouped
@@ -285,11 +286,13 @@ gb_status gb_pool_set_profile_events(gb_pool* pool, int which, void* start_event
 /*
  * Work accounting of the most recent decode/append steps (not part of the method).
  * Synchronises `stream` and copies up to max_steps records, oldest first, into
- * out[n][8] (host): [0] tokens per KV head the per-beam path reads when every
+ * out[n][10] (host): [0] tokens per KV head the per-beam path reads when every
  * beam reads its whole context, [1] the same with shared-prefix segments taken
  * by the grouped path, [2] sum over segments of (query rows of one KV head) x
  * tokens, [3] sum over segments of (128-row tiles) x tokens, [4] segments,
- * [5] 128-row tiles, [6] tokens appended by the step, [7] step index.
+ * [5] 128-row tiles, [6] tokens appended by the step, [7] step index,
+ * [8] sum over segments of their tokens (shared tokens per KV head, each once),
+ * [9] active beams.
  * *n_out receives the number of records (at most the last 4096 steps are kept).
  */
 gb_status gb_pool_read_step_stats(gb_pool* pool, int32_t* out, int max_steps, int* n_out, gb_stream_t stream);

@@ -68,8 +68,9 @@ class OracleRun:
         K, V = self.beam_kv(slot, layer)
         return decode_attention(self.q(layer, slot, pos), K, V, self.wl.attn_scale)
 
-    def decode_step(self, compute: bool = True, slots=None) -> dict | None:
-        """One token per active beam and layer; returns {(layer, slot): o} when compute.
+    def decode_step(self, compute: bool = True, slots=None, layers=None) -> dict | None:
+        """One token per active beam and layer; returns {(layer, slot): o} when compute, for the
+        given slots and layers (default: every active slot and every layer).
 
         Returns None (and changes nothing) when the pool is out of pages.
         """
@@ -86,7 +87,7 @@ class OracleRun:
                 v = self._kv(gen.TAG_KV_V, layer, np.asarray(active, np.uint64), pos)
                 for i, b in enumerate(active):
                     self.kv.append(b, layer, k[i], v[i])
-            if compute:
+            if compute and (layers is None or layer in layers):
                 for b in want:
                     outs[(layer, b)] = self.attention(b, layer, pos)
         self.pos += 1

@@ -21,6 +21,7 @@ GB_ERR_TOO_LARGE = 7
 STATUS_NAMES = {0: "GB_OK", 1: "GB_ERR_INVALID", 2: "GB_ERR_OOM", 3: "GB_ERR_CUDA", 4: "GB_ERR_STATE",
                 5: "GB_ERR_TIMEOUT", 6: "GB_ERR_UNSUPPORTED", 7: "GB_ERR_TOO_LARGE"}
 GB_F32, GB_BF16 = 0, 1
+STATS_WORDS = 10  # words per record of gb_pool_read_step_stats
 GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 
 # Every symbol the header declares, in header order.
@@ -262,9 +263,9 @@ STEP_STATS_FIELDS = ("tokens_per_beam_path", "tokens_with_grouped", "seg_rowtok"
 
 
 def gb_pool_read_step_stats(pool: int, max_steps: int = 4096, stream=None):
-    """Work records of the last steps: an int32 array [n][8] (see include/gambit.h)."""
+    """Work records of the last steps: an int32 array [n][10] (see include/gambit.h)."""
     import numpy as np
-    out = np.zeros((max_steps, 8), dtype=np.int32)
+    out = np.zeros((max_steps, STATS_WORDS), dtype=np.int32)
     n = ctypes.c_int()
     _check(pool, load().gb_pool_read_step_stats(pool, out.ctypes.data, max_steps, ctypes.byref(n),
                                                 stream_handle(stream)), "gb_pool_read_step_stats")

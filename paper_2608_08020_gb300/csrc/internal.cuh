@@ -21,7 +21,7 @@ constexpr int kMaxCowJobs = 1024;
 constexpr int kMaxSegDepth = 16;
 constexpr int kMaxSegRecords = 48;  // grouped partial records per beam (segments x token splits)
 constexpr int kStatsRing = 4096;   // steps kept in the step-stats ring
-constexpr int kStatsWords = 8;   // grouped segments per beam (deeper shared levels use the per-beam path)
+constexpr int kStatsWords = 10;  // words per step record of the step-stats ring
 constexpr int kMlpScratchFloats = 320 * 128 * 128;  // K-split partials of the MLP scorer's first layer (20 MiB)
 
 // Control words at the start of the metadata buffer.
@@ -42,6 +42,7 @@ enum Ctl : int {
   kCtlSegSplit = 13,   // tokens per grouped work unit (segments are split along tokens)
   kCtlGrpNext = 14,    // next grouped work unit to hand out (reset by the grouped kernel's last CTA)
   kCtlGrpDone = 15,    // grouped-kernel CTAs finished (reset by the last one)
+  kCtlSegTok = 16,     // sum over segments of their tokens (the shared tokens the grouped path reads once)
   kCtlWords = 32
 };
 

@@ -235,7 +235,7 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
   __shared__ int tmp[33];
   __shared__ int s_alloc[kMaxBeams];
   __shared__ int s_tail[kMaxBeams];
-  __shared__ int s_ncow;
+  __shared__ int s_ncow, s_nact;
   __shared__ int s_tok[2];
   const int b = threadIdx.x;
   const bool act = b < v.max_beams && v.active[b] != 0;
@@ -267,8 +267,10 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
     need_total = (last_idx >= first_new ? last_idx - first_new + 1 : 0) + (cow ? 1 : 0);
     too_long = last_idx >= v.max_pages;
   }
-  int total_need;
+  int total_need, nact;
   block_exclusive_scan(need_total, tmp, &total_need);
+  block_exclusive_scan(act ? 1 : 0, tmp, &nact);
+  if (b == 0) s_nact = nact;
   const bool any_too_long = __syncthreads_or(too_long);
   if (any_too_long || total_need > v.ctl[kCtlFree]) {
     if (b == 0) v.ctl[kCtlCowJobs] = 0;
@@ -345,6 +347,8 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
     e[5] = v.grouped ? v.ctl[kCtlSegTiles] : 0;
     e[6] = n_tokens;
     e[7] = step;
+    e[8] = v.grouped ? v.ctl[kCtlSegTok] : 0;
+    e[9] = s_nact;
     v.ctl[kCtlSteps] = step + 1;
   }
   if (b == 0) v.ctl[kCtlStepOk] = 1;

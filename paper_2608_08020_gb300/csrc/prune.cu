@@ -219,11 +219,9 @@ __global__ void __launch_bounds__(1024) k_fork_slots(PoolView v, const int* __re
 cudaError_t launch_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const uint8_t* elig,
                                 int32_t* parent_out, uint8_t* pruned_out, uint32_t* lineage_out, cudaStream_t s) {
   const int grid = pool->view.max_beams < pool->num_sms ? pool->view.max_beams : pool->num_sms;
-  prof_begin(pool, GB_PROF_PRUNE, s);
   const int C = pool->capacity > 0 ? pool->capacity : pool->view.max_beams;
   const cudaError_t e = launch_pdl(k_prune_branch, grid, 1024, 0, s, pool->view, C, K, fanout, warmup, elig,
                                    parent_out, pruned_out, reinterpret_cast<unsigned*>(lineage_out));
-  prof_end(pool, GB_PROF_PRUNE, s);
   pool->launches += 1;
   return e;
 }
@@ -240,11 +238,11 @@ extern "C" gb_status gb_fork_slots(gb_pool* pool, const int32_t* parent_of_dev, 
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   prof_begin(pool, GB_PROF_PRUNE, s);
   launch_pdl(k_fork_slots, 1, 1024, 0, s, pool->view, parent_of_dev);
-  prof_end(pool, GB_PROF_PRUNE, s);
   pool->launches += 1;
   gb_status st = check_launch(pool, "fork_slots");
   if (st != GB_OK) return st;
   if (rebuild_segments(pool, s) != cudaSuccess) return check_launch(pool, "segments");
+  prof_end(pool, GB_PROF_PRUNE, s);
   return GB_OK;
 }
 
@@ -264,9 +262,11 @@ extern "C" gb_status gb_prune_branch(gb_pool* pool, int K, int fanout, int warmu
   if (!pool->seeded) return fail(pool, GB_ERR_STATE, "pool not seeded");
   if (pool->next_layer != 0) return fail(pool, GB_ERR_STATE, "prune_branch inside an open step");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  prof_begin(pool, GB_PROF_PRUNE, s);
   launch_prune_branch(pool, K, fanout, warmup, eligible_dev, parent_out_dev, pruned_out_dev, lineage_out_dev, s);
   gb_status st = check_launch(pool, "prune_branch");
   if (st != GB_OK) return st;
   if (rebuild_segments(pool, s) != cudaSuccess) return check_launch(pool, "segments");
+  prof_end(pool, GB_PROF_PRUNE, s);
   return GB_OK;
 }

@@ -137,16 +137,18 @@ __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
   const int nseg = v.ctl[kCtlSegCount];
   const int rows_per_tile = 128;
   const int cap = v.max_beams * kMaxSegRecords;
-  int rowtok = 0, tiletok = 0;
+  int rowtok = 0, tiletok = 0, segtok = 0;
   for (int base = 0; base < nseg; base += blockDim.x) {
     const int s = base + threadIdx.x;
     const int tiles = s < nseg ? (v.seg_g[s] * v.G + rows_per_tile - 1) / rows_per_tile : 0;
     const int toks = s < nseg ? v.seg_len[s] * v.P : 0;
-    int t1, t2;
+    int t1, t2, t3;
     block_exclusive_scan(s < nseg ? v.seg_g[s] * v.G * toks : 0, tmp, &t1);
     block_exclusive_scan(tiles * toks, tmp, &t2);
+    block_exclusive_scan(toks, tmp, &t3);
     rowtok += t1;
     tiletok += t2;
+    segtok += t3;
   }
   if (threadIdx.x == 0) {
     const long long work = (long long)tiletok * v.Hkv;              // tile-tokens over all heads
@@ -160,6 +162,7 @@ __global__ void __launch_bounds__(1024) k_seg_tiles(PoolView v) {
     v.ctl[kCtlSegSplit] = split;
     v.ctl[kCtlSegRowTok] = rowtok;
     v.ctl[kCtlSegTileTok] = tiletok;
+    v.ctl[kCtlSegTok] = segtok;
   }
   __syncthreads();
   const int split = s_split;

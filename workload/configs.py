@@ -113,5 +113,13 @@ MEMORY_CAPPED = Workload(
     hidden=4096, hidden_dtype="bf16", w_scale=1.0 / 64, q_scale=None, attn_scale=1.0 / math.sqrt(128),
     pool_bytes=120 * 10**9)
 
-ALL = {w.name: w for w in (TINY, QWEN3_8B_LAYER, PARALLEL_SAMPLING, LONG_CONTEXT, MEMORY_CAPPED)}
-BY_INDEX = [TINY, QWEN3_8B_LAYER, PARALLEL_SAMPLING, LONG_CONTEXT, MEMORY_CAPPED]
+# No shared KV at all: 64 independent traces of 16384 tokens (a one-token prompt, whose partly
+# filled page every trace but one copies on its first append, and no tournament, so no forks).
+# Every page is read by one beam only: the per-beam path's own roofline.
+UNSHARED = Workload(
+    name="unshared-64beams-L16384", num_layers=1, num_q_heads=32, num_kv_heads=8, head_dim=128,
+    page_size=16, kv_dtype="bf16", beams=64, prompt_len=1, context=16384, interval=1 << 30, K=0, fanout=2,
+    hidden=4096, hidden_dtype="bf16", w_scale=1.0 / 64, q_scale=None, attn_scale=1.0 / math.sqrt(128))
+
+ALL = {w.name: w for w in (TINY, QWEN3_8B_LAYER, PARALLEL_SAMPLING, LONG_CONTEXT, MEMORY_CAPPED, UNSHARED)}
+BY_INDEX = [TINY, QWEN3_8B_LAYER, PARALLEL_SAMPLING, LONG_CONTEXT, MEMORY_CAPPED, UNSHARED]
