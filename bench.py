@@ -247,11 +247,12 @@ def measured_peaks() -> dict:
 def _oracle_worker(wl_dict, slot_hist, positions, barrier, out_q):
     """Spawned process: for each layer, materialise its beams' KV (untimed), then time fp64 decode
     attention of every step; reports the timed seconds summed over layers."""
-    from oracle.attention import decode_attention
+    from oracle import backends
     from oracle.beams import kv_from_history
     from workload import gen
     from workload.configs import Workload
     wl = Workload(**wl_dict)
+    decode_attention = backends.get().decode_attention
     hscale = [gen.head_scales(wl.seed, l, wl.num_kv_heads, *wl.head_scale) for l in range(wl.num_layers)] \
         if wl.head_scale else None
     barrier.wait()
@@ -311,7 +312,8 @@ def oracle_sample(wl, steps: int, sample_beams: int, workers: int | None = None)
     total = t_attn + t_round * steps / wl.interval
     return {"value": beams_done / total, "unit": "beam-tokens/s", "cores": len(chunks), "kind": "oracle",
             "seconds": round(total, 3), "wall_seconds": round(t_attn + t_round, 3),
-            "sample": (f"{steps} steps x {len(sample)} of {wl.beams} beams: fp64 two-pass decode attention at "
+            "sample": (f"{steps} steps x {len(sample)} of {wl.beams} beams: the C++ oracle's fp64 two-pass decode "
+                       f"attention over all {wl.num_layers} layer(s) at "
                        f"L={L} over {len(chunks)} single-threaded spawn processes, plus the fp64 probe over all "
                        f"{wl.beams} beams and one tournament round on the oracle pool every {wl.interval} steps")}
 

@@ -10,6 +10,10 @@ method's arithmetic.
 
 Modules
 -------
+* ``cpp/gambit_oracle.cpp`` - the oracle of the hot path in plain C++17 (attention,
+  probe, running mean, tournament, the pool, beam KV copied on fork), built by
+  ``build_cpp`` and loaded through ``cpp``; ``backends`` selects it (the default) or
+  its numpy twin below, and the oracle tests pin both and check one against the other.
 * ``attention``  - decode attention as its textbook definition (fp64,
   two-pass softmax) over each beam's full, materialised KV.
 * ``probe``      - scorer probe sigma(w.h + b) in fp64 and the running-mean

@@ -40,6 +40,14 @@ class BeamKV:
         self.K[slot][layer] = np.concatenate([self.K[slot][layer], k[None].astype(np.float32)])
         self.V[slot][layer] = np.concatenate([self.V[slot][layer], v[None].astype(np.float32)])
 
+    def append_rows(self, slot: int, layer: int, k: np.ndarray, v: np.ndarray) -> None:
+        """Append n rows k, v [n][Hkv][D] to the slot's layer."""
+        self.K[slot][layer] = np.concatenate([self.K[slot][layer], np.asarray(k, np.float32)])
+        self.V[slot][layer] = np.concatenate([self.V[slot][layer], np.asarray(v, np.float32)])
+
+    def get(self, slot: int, layer: int) -> tuple[np.ndarray, np.ndarray]:
+        return self.K[slot][layer], self.V[slot][layer]
+
     def branch(self, child: int, parent: int) -> None:
         self.K[child] = [a.copy() for a in self.K[parent]]
         self.V[child] = [a.copy() for a in self.V[parent]]

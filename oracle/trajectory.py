@@ -1,12 +1,15 @@
 """Run a workload schedule on the oracle.
 
-Mirrors the schedule of ``workload.configs`` on ``oracle.pool.PoolOracle``:
+Mirrors the schedule of ``workload.configs`` on the oracle's pool (``oracle.cpp.CppPool``, or
+``oracle.pool.PoolOracle`` with the numpy backend):
 seeding, decode steps (every layer), chunked appends, the probe with the
 running-mean update, and tournament rounds.  Attention outputs come from each
-beam's full KV: the literal copy-on-fork arrays (``oracle.beams.BeamKV``) for
+beam's full KV: the literal copy-on-fork arrays (``CppBeamKV`` / ``oracle.beams.BeamKV``) for
 small cases, or the KV rebuilt from the writer history for sampled beams of
 large cases.  Every input is regenerated here from the seeded generator; no
-value is taken from the CUDA path.
+value is taken from the CUDA path.  The arithmetic (attention, probe, running mean,
+tournament, pool) comes from the chosen oracle backend (``oracle.backends``): the C++
+oracle by default, or its numpy twin.
 
 This module is oracle code (test infrastructure), see ``oracle/__init__.py``.
 """
@@ -14,21 +17,20 @@ from __future__ import annotations
 
 import numpy as np
 
-from oracle.attention import decode_attention
-from oracle.beams import BeamKV, kv_from_history
-from oracle.pool import PoolOracle
-from oracle.probe import probe_score, running_mean_update
+from oracle import backends
+from oracle.beams import kv_from_history
 from workload import gen
 from workload.configs import Workload
 
 
 class OracleRun:
     def __init__(self, wl: Workload, literal_kv: bool = True, num_pages: int | None = None,
-                 max_context: int | None = None):
+                 max_context: int | None = None, backend: str | None = None):
         self.wl = wl
-        self.pool = PoolOracle(num_pages if num_pages is not None else wl.pool_pages(max_context), wl.beams,
-                               wl.table_width(max_context), wl.page_size)
-        self.kv = BeamKV(wl.num_layers, wl.beams, wl.num_kv_heads, wl.head_dim) if literal_kv else None
+        self.B = backends.get(backend or backends.DEFAULT)
+        self.pool = self.B.Pool(num_pages if num_pages is not None else wl.pool_pages(max_context), wl.beams,
+                                wl.table_width(max_context), wl.page_size)
+        self.kv = self.B.BeamKV(wl.num_layers, wl.beams, wl.num_kv_heads, wl.head_dim) if literal_kv else None
         self.hscale = None
         if wl.head_scale is not None:
             self.hscale = [gen.head_scales(wl.seed, l, wl.num_kv_heads, *wl.head_scale)
@@ -59,14 +61,14 @@ class OracleRun:
     def beam_kv(self, slot: int, layer: int) -> tuple[np.ndarray, np.ndarray]:
         """The full K, V of a beam: literal arrays when kept, else rebuilt from its writer history."""
         if self.kv is not None:
-            return self.kv.K[slot][layer], self.kv.V[slot][layer]
+            return self.kv.get(slot, layer)
         wl = self.wl
         return kv_from_history(self.pool.history[slot], wl.seed, layer, wl.num_kv_heads, wl.head_dim,
                                wl.kv_dtype, self.hscale[layer] if self.hscale else None)
 
     def attention(self, slot: int, layer: int, pos: int) -> np.ndarray:
         K, V = self.beam_kv(slot, layer)
-        return decode_attention(self.q(layer, slot, pos), K, V, self.wl.attn_scale)
+        return self.B.decode_attention(self.q(layer, slot, pos), K, V, self.wl.attn_scale)
 
     def decode_step(self, compute: bool = True, slots=None, layers=None) -> dict | None:
         """One token per active beam and layer; returns {(layer, slot): o} when compute, for the
@@ -103,10 +105,8 @@ class OracleRun:
             pos = np.arange(self.pos, self.pos + n, dtype=np.uint64)
             for layer in range(wl.num_layers):
                 for b in active:
-                    k = self._kv(gen.TAG_KV_K, layer, b, pos)
-                    v = self._kv(gen.TAG_KV_V, layer, b, pos)
-                    self.kv.K[b][layer] = np.concatenate([self.kv.K[b][layer], k])
-                    self.kv.V[b][layer] = np.concatenate([self.kv.V[b][layer], v])
+                    self.kv.append_rows(b, layer, self._kv(gen.TAG_KV_K, layer, b, pos),
+                                        self._kv(gen.TAG_KV_V, layer, b, pos))
         self.pos += n
 
     def probe_scores(self, slots=None) -> dict:
@@ -114,7 +114,7 @@ class OracleRun:
         wl = self.wl
         slots = [int(b) for b in np.flatnonzero(self.pool.active)] if slots is None else slots
         h = gen.hidden_rows(wl.seed, np.asarray(slots), self.pos, wl.hidden, wl.hidden_dtype)
-        s = probe_score(h, self.w, wl.bias)
+        s = self.B.probe_score(h, self.w, wl.bias)
         return dict(zip(slots, s))
 
     def probe(self, mask=None) -> dict:
@@ -122,7 +122,7 @@ class OracleRun:
         scores = self.probe_scores()
         for b, x in scores.items():
             if mask is None or mask[b]:
-                m, n = running_mean_update(self.pool.mean[b], int(self.pool.nsteps[b]), np.float32(x))
+                m, n = self.B.running_mean_update(self.pool.mean[b], int(self.pool.nsteps[b]), np.float32(x))
                 self.pool.mean[b] = m
                 self.pool.nsteps[b] = n
         return scores
@@ -130,7 +130,8 @@ class OracleRun:
     def push_scores(self, scores32: np.ndarray, mask=None) -> None:
         for b in np.flatnonzero(self.pool.active):
             if mask is None or mask[b]:
-                m, n = running_mean_update(self.pool.mean[b], int(self.pool.nsteps[b]), np.float32(scores32[b]))
+                m, n = self.B.running_mean_update(self.pool.mean[b], int(self.pool.nsteps[b]),
+                                                  np.float32(scores32[b]))
                 self.pool.mean[b] = m
                 self.pool.nsteps[b] = n
 

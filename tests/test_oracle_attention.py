@@ -3,6 +3,19 @@ import numpy as np
 import pytest
 
 from oracle.attention import decode_attention, softmax_weights
+from oracle import backends
+
+NAMES = {'decode_attention': 'decode_attention', 'softmax_weights': 'softmax_weights'}
+
+@pytest.fixture(autouse=True, params=backends.NAMES)
+def oracle_backend(request, monkeypatch):
+    """Every pin runs on both oracles: the C++ one and its numpy twin."""
+    B = backends.get(request.param)
+    monkeypatch.setattr(backends, "DEFAULT", request.param)
+    for name, attr in NAMES.items():
+        monkeypatch.setitem(globals(), name, getattr(B, attr))
+    return B
+
 
 rng = np.random.default_rng(1)
 

@@ -6,8 +6,21 @@ import pytest
 
 from oracle.attention import decode_attention
 from oracle.pool import ERR_INVALID, ERR_OOM, ERR_STATE, PoolOracle
+from oracle import backends
 from oracle.trajectory import OracleRun
 from workload.configs import TINY
+
+NAMES = {'PoolOracle': 'Pool', 'decode_attention': 'decode_attention'}
+
+@pytest.fixture(autouse=True, params=backends.NAMES)
+def oracle_backend(request, monkeypatch):
+    """Every pin runs on both oracles: the C++ one and its numpy twin."""
+    B = backends.get(request.param)
+    monkeypatch.setattr(backends, "DEFAULT", request.param)
+    for name, attr in NAMES.items():
+        monkeypatch.setitem(globals(), name, getattr(B, attr))
+    return B
+
 
 rng = np.random.default_rng(4)
 

@@ -2,8 +2,22 @@
 import math
 
 import numpy as np
+import pytest
 
 from oracle.probe import probe_score, running_mean_update
+from oracle import backends
+
+NAMES = {'probe_score': 'probe_score', 'running_mean_update': 'running_mean_update'}
+
+@pytest.fixture(autouse=True, params=backends.NAMES)
+def oracle_backend(request, monkeypatch):
+    """Every pin runs on both oracles: the C++ one and its numpy twin."""
+    B = backends.get(request.param)
+    monkeypatch.setattr(backends, "DEFAULT", request.param)
+    for name, attr in NAMES.items():
+        monkeypatch.setitem(globals(), name, getattr(B, attr))
+    return B
+
 
 rng = np.random.default_rng(2)
 

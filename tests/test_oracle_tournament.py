@@ -9,6 +9,19 @@ import pytest
 
 from oracle.simulate import simulate
 from oracle.tournament import rank_order, tournament
+from oracle import backends
+
+NAMES = {'rank_order': 'rank_order', 'tournament': 'tournament'}
+
+@pytest.fixture(autouse=True, params=backends.NAMES)
+def oracle_backend(request, monkeypatch):
+    """Every pin runs on both oracles: the C++ one and its numpy twin."""
+    B = backends.get(request.param)
+    monkeypatch.setattr(backends, "DEFAULT", request.param)
+    for name, attr in NAMES.items():
+        monkeypatch.setitem(globals(), name, getattr(B, attr))
+    return B
+
 
 GOLDEN = Path(__file__).parent / "golden"
 
