@@ -227,6 +227,16 @@ gb_status gb_prune_branch(gb_pool* pool, int K, int fanout, int warmup, const ui
                           gb_stream_t stream);
 
 /*
+ * The active slot the tournament would rank last (Algorithm 1, KV saturation: the trace with
+ * the lowest running mean is evicted from the Scheduler view and kept in the Tree view as a
+ * ghost, Section 3.2): NaN means rank last, then the lowest mean, ties to the higher slot -
+ * the ranking of gb_prune_branch read from its end.  Writes the slot to *slot_out_dev (an
+ * int32 device word), or -1 when no slot is active; the caller releases it with gb_release.
+ * Errors: GB_ERR_INVALID for a null pointer.
+ */
+gb_status gb_pool_last_ranked(gb_pool* pool, int32_t* slot_out_dev, gb_stream_t stream);
+
+/*
  * The tree's capacity C (Algorithm 1's C; Section 3.2, Tree view): the
  * tournament takes Case 1 while fewer than C traces are active and Case 2
  * otherwise, and Case 1 never grows the active set beyond C.  Default and

@@ -204,24 +204,34 @@ class CppPool:
     def next_lineage(self) -> int:
         return int(load().gbo_pool_next_lineage(self._h))
 
+    # Tables and histories are copied out of the C++ pool once per state change and cached
+    # (callers index them in loops); every operation that changes them drops the copies.
+    def _changed(self) -> None:
+        self._tables = None
+        self._history = None
+
     @property
     def tables(self) -> list[list[int]]:
-        buf = np.empty(self.max_pages + 1, np.int64)
-        out = []
-        for b in range(self.max_beams):
-            n = load().gbo_pool_table(self._h, b, _ptr(buf), len(buf))
-            out.append([int(p) for p in buf[:n]])
-        return out
+        if getattr(self, "_tables", None) is None:
+            buf = np.empty(self.max_pages + 1, np.int64)
+            out = []
+            for b in range(self.max_beams):
+                n = load().gbo_pool_table(self._h, b, _ptr(buf), len(buf))
+                out.append([int(p) for p in buf[:n]])
+            self._tables = out
+        return self._tables
 
     @property
     def history(self) -> list[list[list[int]]]:
-        out = []
-        for b in range(self.max_beams):
-            n = load().gbo_pool_history(self._h, b, None, 0)
-            buf = np.empty(3 * max(n, 1), np.int64)
-            load().gbo_pool_history(self._h, b, _ptr(buf), n)
-            out.append([[int(buf[3 * i]), int(buf[3 * i + 1]), int(buf[3 * i + 2])] for i in range(n)])
-        return out
+        if getattr(self, "_history", None) is None:
+            out = []
+            for b in range(self.max_beams):
+                n = load().gbo_pool_history(self._h, b, None, 0)
+                buf = np.empty(3 * max(n, 1), np.int64)
+                load().gbo_pool_history(self._h, b, _ptr(buf), n)
+                out.append([[int(buf[3 * i]), int(buf[3 * i + 1]), int(buf[3 * i + 2])] for i in range(n)])
+            self._history = out
+        return self._history
 
     @property
     def cow_events(self) -> list[tuple[int, int, int, int]]:
@@ -247,10 +257,12 @@ class CppPool:
     def seed(self, n_beams: int, prompt_len: int) -> None:
         from oracle.pool import PoolOOM
         assert 1 <= n_beams <= self.max_beams and prompt_len >= 1
+        self._changed()
         if not load().gbo_pool_seed(self._h, int(n_beams), int(prompt_len)):
             raise PoolOOM
 
     def begin_step(self) -> bool:
+        self._changed()
         return bool(load().gbo_pool_begin_step(self._h))
 
     def eligible(self, warmup: int, mask=None) -> np.ndarray:
@@ -265,6 +277,7 @@ class CppPool:
         m = None if mask is None else np.ascontiguousarray(np.asarray(mask) != 0, dtype=np.uint8)
         parent_of = np.empty(self.max_beams, np.int32)
         pruned = np.empty(self.max_beams, np.uint8)
+        self._changed()
         load().gbo_pool_prune_branch(self._h, int(K), int(fanout), int(warmup), None if m is None else _ptr(m),
                                      _ptr(parent_of), _ptr(pruned))
         n_order, n_pruned, n_children = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
@@ -279,10 +292,12 @@ class CppPool:
 
     def fork_slots(self, parent_of) -> None:
         p = np.ascontiguousarray(parent_of, dtype=np.int32)
+        self._changed()
         load().gbo_pool_fork_slots(self._h, _ptr(p))
 
     def release(self, slots) -> None:
         s = np.ascontiguousarray(np.asarray(slots, dtype=np.int64), dtype=np.int32)
+        self._changed()
         load().gbo_pool_release(self._h, _ptr(s) if len(s) else None, len(s))
 
 

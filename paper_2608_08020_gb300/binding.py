@@ -28,7 +28,7 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
            "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
-           "gb_paged_decode_noalloc", "gb_paged_decode_noalloc_status", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_score_mlp", "gb_fork_slots", "gb_scorer_sizes", "gb_scorer_seed",
+           "gb_paged_decode_noalloc", "gb_paged_decode_noalloc_status", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_pool_last_ranked", "gb_score_mlp", "gb_fork_slots", "gb_scorer_sizes", "gb_scorer_seed",
            "gb_scorer_step", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
 GB_PROF_PLAN, GB_PROF_APPEND, GB_PROF_COMBINE, GB_PROF_ATTENTION = 4, 5, 6, 7
@@ -95,6 +95,7 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_paged_decode_noalloc_status": [P, V],
         "gb_pool_read_step_stats": [V, P, I, P, V],
         "gb_pool_set_capacity": [V, I],
+        "gb_pool_last_ranked": [V, V, V],
         "gb_score_mlp": [V, V, I, V, V, V, F, I, V, V, V],
         "gb_fork_slots": [V, V, V],
         "gb_scorer_sizes": [V, P, P, P, P, I, P],
@@ -201,6 +202,10 @@ def gb_prune_branch(pool: int, K: int, fanout: int, warmup: int = 0, eligible=No
 
 def gb_pool_set_capacity(pool: int, capacity: int) -> None:
     _check(pool, load().gb_pool_set_capacity(pool, int(capacity)), "gb_pool_set_capacity")
+
+
+def gb_pool_last_ranked(pool: int, slot_out, stream=None) -> None:
+    _check(pool, load().gb_pool_last_ranked(pool, ptr(slot_out), stream_handle(stream)), "gb_pool_last_ranked")
 
 
 class GbScorerConfig(ctypes.Structure):

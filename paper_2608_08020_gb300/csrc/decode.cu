@@ -519,8 +519,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 
 template <int G>
 __global__ void __launch_bounds__(kMmaWarps * 32, 1)
-    k_decode_mma(PoolView v, const __grid_constant__ CUtensorMap tm, int layer, const __nv_bfloat16* __restrict__ q,
-                 float qscale, int mode, int W) {
+    k_decode_mma(PoolView v, const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtensorMap tmh,
+                 int layer, const __nv_bfloat16* __restrict__ q, float qscale, int mode, int W) {
   pdl_wait();
   pdl_launch_dependents();
   using S = DecodeMmaSmem;
@@ -603,8 +603,11 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 1)
       const int tok = qi.tok0 + qi.i * kChunk;
       const int wrow = ((layer_pages + page) * 2 * v.Hkv + qi.h) * pg8 + ((tok & (v.P - 1)) >> 3);
       const uint32_t bar = bar0 + 8 * stage;
-      mbar_arrive_expect_tx(bar, kMmaStageBytes);
-      tma_chunk(stage0 + stage * kMmaStageBytes, &tm, wrow, bar, pol);
+      // The last chunk of a (beam, head) with at most 8 valid tokens brings only its first
+      // 8-token group (the consumer masks the rest of the stage, whatever it holds).
+      const bool half = qi.i == qi.n - 1 && v.seq_len[qi.b] - tok <= 8;
+      mbar_arrive_expect_tx(bar, half ? kMmaStageBytes / 2 : kMmaStageBytes);
+      tma_chunk(stage0 + stage * kMmaStageBytes, half ? &tmh : &tm, wrow, bar, pol);
     }
   };
 
@@ -895,8 +898,9 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
       wpc = kMmaWarps;
       W = pool->num_sms * kMmaWarps;  // one CTA per SM, as the grouped kernel's split assumes
       e = launch_pdl(k_decode_mma<G>, W / kMmaWarps, kMmaWarps * 32, DecodeMmaSmem::TOTAL, sd, pool->view,
-                     *reinterpret_cast<const CUtensorMap*>(pool->dtmap), layer, static_cast<const __nv_bfloat16*>(q),
-                     qscale, mode, W);
+                     *reinterpret_cast<const CUtensorMap*>(pool->dtmap),
+                     *reinterpret_cast<const CUtensorMap*>(pool->dtmap_half), layer,
+                     static_cast<const __nv_bfloat16*>(q), qscale, mode, W);
     } else {
       e = launch_pdl(k_decode<DT, G>, W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, sd, pool->view, layer, q, qscale,
                      mode, W);

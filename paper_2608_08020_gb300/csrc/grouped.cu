@@ -689,8 +689,12 @@ void make_kv_tensor_maps(gb_pool* pool) {
   }
   if (v.P % 16 == 0) {
     cuuint32_t box[5] = {64, 8, 2, 2, 2};
+    cuuint32_t half[5] = {64, 8, 2, 2, 1};  // the first 8 tokens of a chunk only
     pool->have_dtmap = encode(reinterpret_cast<CUtensorMap*>(pool->dtmap), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, v.kv,
                               dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS &&
+                       encode(reinterpret_cast<CUtensorMap*>(pool->dtmap_half), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5,
+                              v.kv, dims, strides, half, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
   }
 }

@@ -43,6 +43,9 @@ enum Ctl : int {
   kCtlGrpNext = 14,    // next grouped work unit to hand out (reset by the grouped kernel's last CTA)
   kCtlGrpDone = 15,    // grouped-kernel CTAs finished (reset by the last one)
   kCtlSegTok = 16,     // sum over segments of their tokens (the shared tokens the grouped path reads once)
+  kCtlBarCount = 17,   // grid-barrier arrivals of the tournament kernel (only grows)
+  kCtlSegGen = 19,     // segment rebuilds so far (stamps the per-page claim words)
+  kCtlSegAlloc = 20,   // words 20-21: (segments << 32 | member slots) handed out by the running rebuild
   kCtlWords = 32
 };
 
@@ -51,9 +54,8 @@ struct MetaLayout {
   size_t ctl, tables, seq_len, active, gen, nsteps, mean, lineage, refcnt, free_bits;
   size_t plan, cow, partials, total, stats;
   // shared-prefix segments
-  size_t seg_cover, seg_nseg, seg_bstart, seg_bpage, seg_owner, seg_id, seg_i0, seg_len, seg_rep, seg_g,
-      seg_mem_off, seg_fill, seg_members, seg_tile_seg, seg_tile_t, grec, seg_bid, seg_rec_off, seg_nrec,
-      seg_splits, seg_tile_split;
+  size_t seg_cover, seg_nseg, seg_owner, seg_i0, seg_len, seg_rep, seg_g, seg_mem_off, seg_fill, seg_members,
+      seg_tile_seg, seg_tile_t, grec, seg_bid, seg_rec_off, seg_nrec, seg_splits, seg_tile_split, seg_hist;
   int words;            // free-bitmap words
   size_t mlp_scratch;   // MLP scorer partial sums
   int partial_records;  // split-KV partial records
@@ -85,10 +87,7 @@ struct PoolView {
   int group_min;        // segments need at least this many sharing beams
   int* seg_cover;       // [max_beams] leading full pages of the beam covered by segments
   int* seg_nseg;        // [max_beams] segments the beam belongs to (by depth)
-  int* seg_bstart;      // [max_beams][kMaxSegDepth] first table index of the beam's k-th segment
-  int* seg_bpage;       // [max_beams][kMaxSegDepth] page id at that index
-  unsigned long long* seg_owner;  // [num_pages] (rebuild gen << 32 | ~lowest beam) at segment-start pages
-  int* seg_id;          // [num_pages] segment id of a segment-start page
+  unsigned long long* seg_owner;  // [num_pages] claim word of a segment-start page: (rebuild gen << 32) | (segment id + 1)
   int* seg_i0;          // [segments] first table index
   int* seg_len;         // [segments] pages
   int* seg_rep;         // [segments] a member beam whose table lists the pages
@@ -103,6 +102,7 @@ struct PoolView {
   int* seg_bid;         // [max_beams][kMaxSegDepth] segment id of the beam's k-th segment
   int* seg_rec_off;     // [max_beams][kMaxSegDepth] first grouped record of that segment
   int* seg_nrec;        // [max_beams] grouped records of the beam
+  int* seg_hist;        // [2][256] work units per length bucket, and units placed per bucket (rebuild scratch)
   int num_sms;          // multiprocessors (sizes the grouped work split)
   float* grec;          // [max_beams][kMaxSegDepth][Hkv] grouped partial records
   int* stats;           // [kStatsRing][kStatsWords] work of recent steps (see gb_pool_read_step_stats)
@@ -264,10 +264,10 @@ struct gb_pool {
   bool seeded;
   int group_min;
   int capacity = 0;   // the tree's capacity C for the tournament (0: max_beams)
-  unsigned long long seg_gen = 0;           // segment rebuilds so far
   alignas(64) unsigned char tmap[128];      // CUtensorMap over the KV pool (grouped path)
   bool have_tmap = false;
   alignas(64) unsigned char dtmap[128];     // CUtensorMap over the KV pool (per-beam bf16 path)
+  alignas(64) unsigned char dtmap_half[128];  // the same with an 8-token box (short tail chunks)
   bool have_dtmap = false;
   int tmap_oob = 0;                          // first row group past the tensor map (loads zeros)
   std::string last_error;

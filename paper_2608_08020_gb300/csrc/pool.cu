@@ -44,10 +44,7 @@ MetaLayout meta_layout(const gb_pool_config& c) {
   const size_t BD = B * kMaxSegDepth;
   m.seg_cover = take(B * sizeof(int));
   m.seg_nseg = take(B * sizeof(int));
-  m.seg_bstart = take(BD * sizeof(int));
-  m.seg_bpage = take(BD * sizeof(int));
   m.seg_owner = take((size_t)c.num_pages * sizeof(unsigned long long));
-  m.seg_id = take((size_t)c.num_pages * sizeof(int));
   m.seg_i0 = take(BD * sizeof(int));
   m.seg_len = take(BD * sizeof(int));
   m.seg_rep = take(BD * sizeof(int));
@@ -63,6 +60,7 @@ MetaLayout meta_layout(const gb_pool_config& c) {
   m.seg_nrec = take(B * sizeof(int));
   m.seg_splits = take(BD * sizeof(int));
   m.seg_tile_split = take(B * kMaxSegRecords * sizeof(int));
+  m.seg_hist = take(2 * 256 * sizeof(int));
   m.stats = take((size_t)kStatsRing * kStatsWords * sizeof(int));
   m.mlp_scratch = take((size_t)kMlpScratchFloats * sizeof(float));
   m.total = o;
@@ -527,10 +525,7 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   v.record_floats = L.record_floats;
   v.seg_cover = reinterpret_cast<int*>(m + L.seg_cover);
   v.seg_nseg = reinterpret_cast<int*>(m + L.seg_nseg);
-  v.seg_bstart = reinterpret_cast<int*>(m + L.seg_bstart);
-  v.seg_bpage = reinterpret_cast<int*>(m + L.seg_bpage);
   v.seg_owner = reinterpret_cast<unsigned long long*>(m + L.seg_owner);
-  v.seg_id = reinterpret_cast<int*>(m + L.seg_id);
   v.seg_i0 = reinterpret_cast<int*>(m + L.seg_i0);
   v.seg_len = reinterpret_cast<int*>(m + L.seg_len);
   v.seg_rep = reinterpret_cast<int*>(m + L.seg_rep);
@@ -546,6 +541,7 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   v.seg_nrec = reinterpret_cast<int*>(m + L.seg_nrec);
   v.seg_splits = reinterpret_cast<int*>(m + L.seg_splits);
   v.seg_tile_split = reinterpret_cast<int*>(m + L.seg_tile_split);
+  v.seg_hist = reinterpret_cast<int*>(m + L.seg_hist);
   v.num_sms = p->num_sms;
   v.stats = reinterpret_cast<int*>(m + L.stats);
   v.mlp_scratch = reinterpret_cast<float*>(m + L.mlp_scratch);

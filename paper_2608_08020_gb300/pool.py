@@ -76,6 +76,10 @@ class BeamPool:
     def set_capacity(self, capacity: int):
         B.gb_pool_set_capacity(self.handle, capacity)
 
+    def last_ranked(self, out, stream=None):
+        """The active slot the tournament ranks last, written to the int32 device tensor `out` (-1: none)."""
+        B.gb_pool_last_ranked(self.handle, out, stream)
+
     def release(self, slots, stream=None):
         B.gb_release(self.handle, slots, int(slots.numel()), stream)
 

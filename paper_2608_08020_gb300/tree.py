@@ -136,6 +136,7 @@ class TournamentLoop:
         self.target = np.zeros(cfg.max_beams, dtype=np.int64)   # completion length in generated tokens
         self.tree = TreeView(C)
         self.evictions = 0
+        self.victim = torch.zeros(1, dtype=torch.int32, device=self.dev)   # slot chosen by gb_pool_last_ranked
 
     def _append(self) -> bool:
         """One thought for every running trace; False (and nothing appended) if the pool ran
@@ -145,14 +146,14 @@ class TournamentLoop:
         return self.pool.status() == 0
 
     def _evict_lowest(self) -> None:
-        """Memory pressure: the running trace with the lowest mean becomes a ghost (Alg. 1, Section 3.2)."""
-        st = self.pool.read_state()
-        m = np.asarray(st["mean"], dtype=np.float32)
-        # The tournament's ranking (mean descending, ties to the lower slot, NaN last); evict its last.
-        order = sorted(self.tree.slot_node, key=lambda s: (bool(np.isnan(m[s])), 0.0 if np.isnan(m[s]) else -float(m[s]), s))
-        victim = order[-1]
+        """Memory pressure: the running trace with the lowest mean becomes a ghost (Alg. 1, Section 3.2).
+        The device picks it (the tournament's ranking read from its end) and releases it; the
+        host reads back only the slot id, for the Tree view."""
+        self.pool.last_ranked(self.victim)
+        self.pool.release(self.victim)
+        victim = int(self.victim.item())
+        assert victim in self.tree.slot_node, (victim, "the pool's active slots are the running traces")
         self.tree.finish([victim], self.length, GHOST)
-        self.pool.release(torch.tensor([victim], dtype=torch.int32, device=self.dev))
         self.evictions += 1
         self.pool.set_capacity(self.C - self.tree.count(GHOST))
 

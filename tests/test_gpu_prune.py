@@ -86,3 +86,29 @@ def test_large_pool_random_trees(cuda):
         g.append(37 + 16 * r)
         o.append(37 + 16 * r)
     assert g.pool.status() == 0
+
+
+@pytest.mark.parametrize("scores", [
+    [0.5, 0.5, np.nan, 0.25, 0.5, np.nan, 0.0, -0.0],   # NaN ranks last: the higher NaN slot
+    [0.5, 0.1, 0.3, 0.1, 0.9, 0.1, 0.2, 0.7],           # ties on the lowest mean: the higher slot
+    [0.0, -0.0, 0.25, 0.0, 0.5, 0.75, -0.0, 1.0],       # +0 and -0 tie
+])
+def test_last_ranked_is_the_tournaments_last(cuda, scores):
+    """gb_pool_last_ranked (the eviction victim) is the last slot of the oracle's tournament order,
+    also after a release leaves a slot inactive."""
+    import torch
+    from oracle import backends
+    wl = dataclasses.replace(TINY, context=400)
+    g, o = _setup(wl)
+    s = np.array(scores, np.float32)
+    g.pool.push_scores(torch.from_numpy(s).to(g.dev))
+    o.push_scores(s, None)
+    out = torch.full((1,), -7, dtype=torch.int32, device=g.dev)
+    for released in ([], [int(backends.get().rank_order(o.pool.mean, o.pool.active)[-1])]):
+        if released:
+            g.pool.release(torch.tensor(released, dtype=torch.int32, device=g.dev))
+            o.pool.release(released)
+        g.pool.last_ranked(out)
+        want = backends.get().rank_order(o.pool.mean, o.pool.active)[-1]
+        assert int(out.item()) == want, (scores, released)
+    assert g.pool.status() == 0
