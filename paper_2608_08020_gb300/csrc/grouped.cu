@@ -39,8 +39,8 @@
 //
 // Shared memory (dynamic only, 1024-byte aligned, 128-byte swizzle everywhere):
 //   Q     two [128 rows][64 dims] blocks (K-major A operand)                32 KiB
-//   K     3 stages x 16 row groups of 8 tokens: [group][half of D][8][64]    96 KiB
-//   V     3 stages, the same layout                                          96 KiB
+//   K     kKStages (3) stages x 16 row groups of 8 tokens: [group][half of D][8][64]    96 KiB
+//   V     kVStages (3) stages, the same layout                                          96 KiB
 //   xch   row maxima (and at a unit's end the sums) of both groups, per tile parity  2 KiB
 // In a stage the 8-token groups sit 2048 bytes apart, the second half of D at +1024:
 // Q.K^T reads K as the K-major B operand (SBO 2048), P.V reads V as the MN-major B
@@ -66,7 +66,13 @@ namespace {
 constexpr int kRows = 128;     // query rows per tile (MMA M)
 constexpr int kTok = 128;      // tokens per K/V tile (MMA N of Q.K^T)
 constexpr int kHalf = 64;      // tokens per softmax group (MMA K of one P.V)
-constexpr int kStages = 3;
+#ifndef GB_GROUPED_KSTAGES
+#define GB_GROUPED_KSTAGES 3  // K ring depth (a K slot is free once S has read it)
+#endif
+#ifndef GB_GROUPED_VSTAGES
+#define GB_GROUPED_VSTAGES 3  // V ring depth (a V slot is held through the softmax and P.V)
+#endif
+constexpr int kKStages = GB_GROUPED_KSTAGES, kVStages = GB_GROUPED_VSTAGES;
 constexpr int kThreads = 352;
 constexpr int kProducerWarp = 8;     // K producer, unit scheduling, Q gather
 constexpr int kMmaWarp = 9;
@@ -77,18 +83,18 @@ constexpr uint32_t kTmemO = 384;
 
 constexpr int kQ = 0;                // 32 KiB
 constexpr int kHalfStage = 32768;    // K (or V) of one 128-token tile of one head
-constexpr int kKRing = 32768;        // kStages x 32 KiB
-constexpr int kVRing = kKRing + kStages * kHalfStage;
-constexpr int kBar = kVRing + kStages * kHalfStage;  // mbarriers and control words
+constexpr int kKRing = 32768;        // kKStages x 32 KiB
+constexpr int kVRing = kKRing + kKStages * kHalfStage;
+constexpr int kBar = kVRing + kVStages * kHalfStage;  // mbarriers and control words
 constexpr int kXch = kBar + 512;     // float [2 tile parities][2 groups][128 rows]
 constexpr int kSmem = kXch + 2048;
 
 // Control area (8-byte mbarriers, then words).
-constexpr int kBarKFull = 0;         // [kStages]
-constexpr int kBarKEmpty = kBarKFull + 8 * kStages;
-constexpr int kBarVFull = kBarKEmpty + 8 * kStages;
-constexpr int kBarVEmpty = kBarVFull + 8 * kStages;
-constexpr int kBarQFull = kBarVEmpty + 8 * kStages;
+constexpr int kBarKFull = 0;         // [kKStages]
+constexpr int kBarKEmpty = kBarKFull + 8 * kKStages;
+constexpr int kBarVFull = kBarKEmpty + 8 * kKStages;  // [kVStages]
+constexpr int kBarVEmpty = kBarVFull + 8 * kVStages;
+constexpr int kBarQFull = kBarVEmpty + 8 * kVStages;
 constexpr int kBarQEmpty = kBarQFull + 8;
 constexpr int kBarSFull = kBarQEmpty + 8;            // [kSBufs]
 constexpr int kBarPFull = kBarSFull + 8 * kSBufs;    // [kSBufs]
@@ -168,9 +174,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t ctl = sbase + kBar;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + kBar + kWordAbort);
   if (tid == 0) {
-    for (int i = 0; i < kStages; ++i) {
+    for (int i = 0; i < kKStages; ++i) {
       mbar_init(ctl + kBarKFull + 8 * i, 1);
       mbar_init(ctl + kBarKEmpty + 8 * i, 1);
+    }
+    for (int i = 0; i < kVStages; ++i) {
       mbar_init(ctl + kBarVFull + 8 * i, 1);
       mbar_init(ctl + kBarVEmpty + 8 * i, 1);
     }
@@ -217,6 +225,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // read the unit that slot held before.
     int pending = 0;
     if (lane == 0) pending = atomicAdd(&v.ctl[kCtlGrpNext], 1);
+    // The next unit's description is loaded while this unit's second tile is issued, so at
+    // the unit boundary only its page ids and member rows (loaded together) are waited for.
+    Unit xn{};
+    bool have_xn = false;
     for (;; ++uidx) {
       if (!ok || *abort_flag) break;
       const long long u = __shfl_sync(0xffffffffu, pending, 0);
@@ -231,10 +243,30 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive(ctl + kBarSchedFull + 8 * k);
       }
       if (u >= units) break;
-      const Unit x = load_unit(v, u);
+      const Unit x = have_xn ? xn : load_unit(v, u);
+      have_xn = false;
+      // Query rows of the unit: row r = (member, query head of this KV head); lane l takes rows
+      // l, l + 32, l + 64, l + 96.  Their member beams are loaded now, beside the first page ids.
+      const char* qrow[kRows / 32];
+      bool qvalid[kRows / 32];
+#pragma unroll
+      for (int i = 0; i < kRows / 32; ++i) {
+        const int r = lane + 32 * i;
+        const int m = x.t * members_per_tile + r / G, gg = r % G;
+        qvalid[i] = m < x.g;
+        const int b = qvalid[i] ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
+        qrow[i] = reinterpret_cast<const char*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
+      }
       int page_l = 0;
       for (int j = 0; j < x.ntok; ++j, ++n) {
-        const uint32_t st = n % kStages;
+        if (j == 1) {  // prefetch the next unit's description (its id came back with this unit)
+          const long long un = __shfl_sync(0xffffffffu, pending, 0);
+          if (un < units) {
+            xn = load_unit(v, un);
+            have_xn = true;
+          }
+        }
+        const uint32_t st = n % kKStages;
         const int pb = j * ppt;  // first page of the tile within the unit
         if ((pb & 31) == 0) {
           const int tl = (pb + lane) * v.P;
@@ -255,8 +287,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             w = (int)(slab * v.P / 8);
           }
         }
-        if (lane == 0 && n >= (uint32_t)kStages)
-          ok = wait_or_abort(ctl + kBarKEmpty + 8 * st, ((n / kStages) - 1) & 1, abort_flag);
+        if (lane == 0 && n >= (uint32_t)kKStages)
+          ok = wait_or_abort(ctl + kBarKEmpty + 8 * st, ((n / kKStages) - 1) & 1, abort_flag);
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         if (!ok) break;
         const uint32_t bar = ctl + kBarKFull + 8 * st;
@@ -275,20 +307,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             ++n;
             break;
           }
-          // Lane l takes rows l, l + 32, l + 64, l + 96: their member beams first, then all
-          // 64 16-byte pieces of its rows as asynchronous copies into the swizzled layout,
-          // so the whole 32 KiB is in flight at once; rows past the members are zeroed.
-          const char* qrow[kRows / 32];
-          bool qvalid[kRows / 32];
-#pragma unroll
-          for (int i = 0; i < kRows / 32; ++i) {
-            const int r = lane + 32 * i;
-            const int m = x.t * members_per_tile + r / G, gg = r % G;
-            qvalid[i] = m < x.g;
-            const int b = qvalid[i] ? v.seg_members[x.moff + m] / kMaxSegDepth : 0;
-            qrow[i] = reinterpret_cast<const char*>(q + ((size_t)b * v.Hq + (size_t)x.h * G + gg) * 128);
-          }
-          // Query rows are read by every unit of their beams: keep them in L2 against the
+          // All 64 16-byte pieces of the lane's rows go out as asynchronous copies into the
+          // swizzled layout, so the whole 32 KiB is in flight at once; rows past the members
+          // are zeroed.  Query rows are read by every unit of their beams: keep them in L2 against the
           // stream of K/V tiles (evict-last).
           const uint64_t qpol = policy_evict_last();
 #pragma unroll
@@ -312,8 +333,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     // Drain: copies still in flight land before the CTA leaves (bounded).
     if (lane == 0 && *abort_flag) {
-      for (uint32_t k = n > (uint32_t)kStages ? n - kStages : 0; k < n; ++k)
-        mbar_wait_bounded(ctl + kBarKFull + 8 * (k % kStages), (k / kStages) & 1, kWaitLimitNs / 8);
+      for (uint32_t k = n > (uint32_t)kKStages ? n - kKStages : 0; k < n; ++k)
+        mbar_wait_bounded(ctl + kBarKFull + 8 * (k % kKStages), (k / kKStages) & 1, kWaitLimitNs / 8);
     }
   } else if (warp == kVProducerWarp) {
     // ------------------------------------------------------------------ V producer
@@ -333,7 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Unit x = load_unit(v, id);
       int page_l = 0;
       for (int j = 0; j < x.ntok; ++j, ++n) {
-        const uint32_t st = n % kStages;
+        const uint32_t st = n % kVStages;
         const int pb = j * ppt;
         if ((pb & 31) == 0) {
           const int tl = (pb + lane) * v.P;
@@ -350,8 +371,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             w = (int)(slab * v.P / 8);
           }
         }
-        if (lane == 0 && n >= (uint32_t)kStages)
-          ok = wait_or_abort(ctl + kBarVEmpty + 8 * st, ((n / kStages) - 1) & 1, abort_flag);
+        if (lane == 0 && n >= (uint32_t)kVStages)
+          ok = wait_or_abort(ctl + kBarVEmpty + 8 * st, ((n / kVStages) - 1) & 1, abort_flag);
         ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
         if (!ok) break;
         const uint32_t bar = ctl + kBarVFull + 8 * st;
@@ -361,8 +382,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (lane == 0 && *abort_flag) {
-      for (uint32_t k = n > (uint32_t)kStages ? n - kStages : 0; k < n; ++k)
-        mbar_wait_bounded(ctl + kBarVFull + 8 * (k % kStages), (k / kStages) & 1, kWaitLimitNs / 8);
+      for (uint32_t k = n > (uint32_t)kVStages ? n - kVStages : 0; k < n; ++k)
+        mbar_wait_bounded(ctl + kBarVFull + 8 * (k % kVStages), (k / kVStages) & 1, kWaitLimitNs / 8);
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------------ MMA issuer
@@ -390,11 +411,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         j_s = 0;
       }
       if (j_s == 0 && !mbar_test(ctl + kBarQFull, uidx_s & 1)) return false;
-      if (!mbar_test(ctl + kBarKFull + 8 * (n_s % kStages), (n_s / kStages) & 1)) return false;
+      if (!mbar_test(ctl + kBarKFull + 8 * (n_s % kKStages), (n_s / kKStages) & 1)) return false;
       return n_pv + (kSBufs - 1) >= n_s;
     };
     auto issue_s = [&]() {
-      const uint32_t st = n_s % kStages, sb = n_s % kSBufs;
+      const uint32_t st = n_s % kKStages, sb = n_s % kSBufs;
       tc_fence_after();
       const uint32_t kb = sbase + kKRing + st * kHalfStage;
 #pragma unroll
@@ -436,11 +457,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             progressed = true;
           }
         }
-        const uint32_t pb = n_pv % kSBufs, st = n_pv % kStages;
+        const uint32_t pb = n_pv % kSBufs, st = n_pv % kVStages;
         // P.V(n) needs both groups' P; a unit's first P.V also needs the previous unit's
         // accumulator read out (o_free), since it overwrites it.
         if (have_p && n_pv < n_s && mbar_test(ctl + kBarPFull + 8 * pb, (n_pv / kSBufs) & 1) &&
-            mbar_test(ctl + kBarVFull + 8 * st, (n_pv / kStages) & 1) &&
+            mbar_test(ctl + kBarVFull + 8 * st, (n_pv / kVStages) & 1) &&
             (j_p > 0 || uidx_p == 0 || mbar_test(ctl + kBarOFree, (uidx_p - 1) & 1))) {
           tc_fence_after();
           const uint32_t vb = sbase + kVRing + st * kHalfStage;

@@ -252,26 +252,31 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
       if (a.pruned_out) a.pruned_out[tid] = s_pruned[tid];
       if (a.lineage_out) a.lineage_out[tid] = k >= 0 ? lin0 + k : v.lineage[tid];
     }
-    // Fork: this CTA's parents.  For table index i of parent p, each child c either already
-    // holds page tp[i] (nothing changes) or drops its old page and takes tp[i]; the new
-    // references of one parent's page are added at once.
-    for (int j = blockIdx.x; j < npar; j += gridDim.x) {
+    // Fork: this CTA's parents, each by its own group of threads (ppc parents at a time).  For
+    // table index i of parent p, each child c either already holds page tp[i] (nothing
+    // changes) or drops its old page and takes tp[i]; the new references of one parent's page
+    // are added at once.
+    const int mine = npar > (int)blockIdx.x ? (npar - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+    int ppc = 1;
+    while (ppc < 32 && ppc < mine) ppc <<= 1;
+    const int tpp = kTourThreads / ppc, fg = tid / tpp, ft = tid % tpp;
+    for (int j = blockIdx.x + fg * gridDim.x; j < npar; j += ppc * gridDim.x) {
       const int p = blist[j];
       const int k0 = j * per, k1 = min(k0 + per, nchild);
       const int new_n = (v.seq_len[p] + v.P - 1) / v.P;
       int m = new_n;
       for (int c = k0; c < k1; ++c) {
-        const int s = cslot[c];
-        m = max(m, s_act[s] ? (v.seq_len[s] + v.P - 1) / v.P : 0);
+        const int sl = cslot[c];
+        m = max(m, s_act[sl] ? (v.seq_len[sl] + v.P - 1) / v.P : 0);
       }
       const int* tp = v.tables + (size_t)p * v.max_pages;
-      for (int i = tid; i < m; i += blockDim.x) {
+      for (int i = ft; i < m; i += tpp) {
         const int nw = i < new_n ? tp[i] : -1;
         int add = 0;
         for (int c = k0; c < k1; ++c) {
-          const int s = cslot[c];
-          const int old_n = s_act[s] ? (v.seq_len[s] + v.P - 1) / v.P : 0;
-          int* ts = v.tables + (size_t)s * v.max_pages;
+          const int sl = cslot[c];
+          const int old_n = s_act[sl] ? (v.seq_len[sl] + v.P - 1) / v.P : 0;
+          int* ts = v.tables + (size_t)sl * v.max_pages;
           const int old = i < old_n ? ts[i] : -1;
           if (old == nw) continue;
           if (nw >= 0) ++add;
@@ -280,18 +285,21 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
         }
         if (add > 0) atomicAdd(&v.refcnt[nw], add);
       }
-      __syncthreads();  // every thread has read the children's old lengths
-      if (tid < k1 - k0) {
-        const int c = k0 + tid, s = cslot[c];
-        v.seq_len[s] = v.seq_len[p];
-        v.mean[s] = v.mean[p];
-        v.nsteps[s] = v.nsteps[p];
-        v.gen[s] = 0;
-        v.active[s] = 1;
-        v.lineage[s] = lin0 + c;
-      }
-      __syncthreads();
     }
+    __syncthreads();  // every thread has read the children's old lengths
+    // The children's per-slot state, for the parents this CTA forked.
+    for (int c = tid; c < nchild; c += blockDim.x) {
+      const int j = c / per;
+      if (j % (int)gridDim.x != (int)blockIdx.x) continue;
+      const int sl = cslot[c], p = blist[j];
+      v.seq_len[sl] = v.seq_len[p];
+      v.mean[sl] = v.mean[p];
+      v.nsteps[sl] = v.nsteps[p];
+      v.gen[sl] = 0;
+      v.active[sl] = 1;
+      v.lineage[sl] = lin0 + c;
+    }
+    __syncthreads();
     if (tid == 0 && s_freed > 0) {
       atomicAdd(&v.ctl[kCtlFree], s_freed);
       atomicMin(&v.ctl[kCtlCursor], s_minword);
