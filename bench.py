@@ -559,7 +559,6 @@ def run_ours(args) -> None:
         for l in range(NL):
             if prof is not None:
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_DECODE, *(prof["dec"][l] if "dec" in prof else (None, None)))
-                B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_GROUPED, *(prof["gr"][l] if "gr" in prof else (None, None)))
                 B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_ATTENTION, *(prof["att"][l] if "att" in prof else (None, None)))
                 if "app" in prof:
                     B.gb_pool_set_profile_events(pool.handle, B.GB_PROF_APPEND, *prof["app"][l])
@@ -711,8 +710,7 @@ def run_ours(args) -> None:
     # Each event record splits the step's chain of programmatically dependent launches, so the
     # kernel durations come from these steps and the timed window below carries no such records.
     pl = list(steps_of("profile"))
-    profs = {i: {"dec": [ev_pair() for _ in range(NL)], "gr": [ev_pair() for _ in range(NL)],
-                 "att": [ev_pair() for _ in range(NL)]} for i in pl}
+    profs = {i: {"dec": [ev_pair() for _ in range(NL)], "att": [ev_pair() for _ in range(NL)]} for i in pl}
     if args.breakdown:
         for i in pl:
             profs[i].update({"app": [ev_pair() for _ in range(NL)], "comb": [ev_pair() for _ in range(NL)],
@@ -735,15 +733,13 @@ def run_ours(args) -> None:
     stats = B.gb_pool_read_step_stats(pool.handle, max_steps=len(pl))   # one record per profiled step
     assert len(stats) == len(pl), (len(stats), len(pl))
     dec_ms = [a.elapsed_time(b) for i in pl for a, b in profs[i]["dec"]]
-    gr_ms = [a.elapsed_time(b) for i in pl for a, b in profs[i]["gr"]]
     att_ms = [a.elapsed_time(b) for i in pl for a, b in profs[i]["att"]]
     step_kernels_us = None
     if args.breakdown:
         step_kernels_us = {
             "plan": statistics.mean(profs[i]["plan"][0].elapsed_time(profs[i]["plan"][1]) for i in pl) * 1e3,
             "append": statistics.mean(a.elapsed_time(b) for i in pl for a, b in profs[i]["app"]) * 1e3,
-            "grouped": statistics.mean(gr_ms) * 1e3,
-            "decode": statistics.mean(dec_ms) * 1e3,
+            "attention": statistics.mean(dec_ms) * 1e3,
             "combine": statistics.mean(a.elapsed_time(b) for i in pl for a, b in profs[i]["comb"]) * 1e3,
         }
 
@@ -802,14 +798,17 @@ def run_ours(args) -> None:
     fork_us = statistics.mean(rprof[i]["fork"][0].elapsed_time(rprof[i]["fork"][1]) for i in timed_rounds) * 1e3 \
         if (timed_rounds and seq is not None) else None
     grouped_on = flags != B.GB_PATH_PER_BEAM and wl.kv_dtype == "bf16" and D == 128
-    # The per-beam kernel: warp-level MMAs for bf16 pools with 128-dim heads, paired fp32 FMAs otherwise.
+    # The attention launch of a layer-step: k_attention (the grouped tcgen05 role over shared
+    # segments and the warp-MMA per-beam role over the tails) on the grouped path; the per-beam
+    # kernel alone otherwise (warp-level MMAs for bf16 pools with 128-dim heads, paired fp32 FMAs
+    # else).
     dec = "k_decode_mma" if wl.kv_dtype == "bf16" and D == 128 else "k_decode"
 
     # Algorithmic work per launch, from the library's per-step records of the profiled steps:
-    #   per-beam kernel: the tokens it reads (all KV heads, K and V) + the queries;
-    #   k_grouped: unique bytes = every shared segment's pages once (K and V of every KV head);
-    #              bytes_read = the K/V tiles it reads (once per 128-row query tile);
-    #              useful flops = 4 * D per (query row, token) for Q.K^T and P.V.
+    #   per-beam role: the tokens it reads (all KV heads, K and V) + the queries;
+    #   grouped role: unique bytes = every shared segment's pages once (K and V of every KV head);
+    #                 bytes_read = the K/V tiles it reads (once per 128-row query tile);
+    #                 useful flops = 4 * D per (query row, token) for Q.K^T and P.V.
     esz = 2 if wl.kv_dtype == "bf16" else 4
     kv_tok = 2 * Hkv * D * esz
     q_bytes = C * Hq * D * esz
@@ -820,8 +819,7 @@ def run_ours(args) -> None:
     gr_unique = statistics.mean(int(s[8]) * kv_tok for s in stats) if grouped_on else 0.0
     gr_flops = statistics.mean(Hkv * int(s[2]) * 4 * D for s in stats) if grouped_on else 0.0
     dec_avg_s = statistics.mean(dec_ms) / 1e3
-    gr_avg_s = statistics.mean(gr_ms) / 1e3 if grouped_on else 0.0
-    achieved = dec_bytes / dec_avg_s / 1e9
+    att_avg_s = statistics.mean(att_ms) / 1e3
     peaks = measured_peaks()
     peak = peaks.get("hbm_gbs")
     peak_src = "measured" if peak else "fallback"
@@ -829,30 +827,29 @@ def run_ours(args) -> None:
     tpeak = peaks.get("bf16_tflops_sustained") or peaks.get("bf16_tflops")
     tpeak_src = "measured sustained" if tpeak else "fallback"
     tpeak = tpeak or 1700.0
-    kernels = {dec: {"us": dec_avg_s * 1e6, "bytes": dec_bytes, "gbps": achieved, "frac_hbm": achieved / peak}}
-    if grouped_on and gr_avg_s > 0:
-        kernels["k_grouped"] = {"us": gr_avg_s * 1e6, "bytes": gr_unique, "bytes_read": gr_read,
-                                "gbps": gr_unique / gr_avg_s / 1e9, "frac_hbm": gr_unique / gr_avg_s / 1e9 / peak,
-                                "gbps_read": gr_read / gr_avg_s / 1e9, "flops": gr_flops,
-                                "tflops": gr_flops / gr_avg_s / 1e12, "frac_tensor": gr_flops / gr_avg_s / 1e12 / tpeak,
-                                "segments": statistics.mean(int(s[4]) for s in stats),
-                                "work_units": statistics.mean(int(s[5]) * Hkv for s in stats)}
-    att_avg_s = statistics.mean(att_ms) / 1e3
-    if "k_grouped" in kernels:
-        # The grouped and per-beam kernels form one phase of the step (they run side by side, or
-        # back to back on two streams), timed from before the fork to after the join.
-        pair_bytes = gr_unique + dec_bytes
-        tr = captured_traffic("k_grouped+" + dec, wl.name, args.flags, pair_bytes)
-        roofline = {"bound": "hbm", "kernel": f"k_grouped + {dec} (the attention phase)",
-                    "achieved": pair_bytes / att_avg_s / 1e9, "peak": peak, "unit": "GB/s",
-                    "frac": pair_bytes / att_avg_s / 1e9 / peak, "traffic": tr, "bytes_per_launch": pair_bytes,
-                    "bytes_read_per_launch": gr_read + dec_bytes, "phase_us": att_avg_s * 1e6,
-                    "peak_source": f"{peak_src} hbm_gbs"}
+    if grouped_on:
+        kname = "k_attention"
+        k_bytes = gr_unique + dec_bytes
+        achieved = k_bytes / dec_avg_s / 1e9
+        kernels = {kname: {"us": dec_avg_s * 1e6, "bytes": k_bytes, "gbps": achieved, "frac_hbm": achieved / peak,
+                           "bytes_read": gr_read + dec_bytes,
+                           "grouped_role": {"bytes": gr_unique, "bytes_read": gr_read, "flops": gr_flops,
+                                            "tflops_over_launch": gr_flops / dec_avg_s / 1e12,
+                                            "frac_tensor_over_launch": gr_flops / dec_avg_s / 1e12 / tpeak,
+                                            "tensor_peak_source": tpeak_src,
+                                            "segments": statistics.mean(int(s[4]) for s in stats),
+                                            "work_units": statistics.mean(int(s[5]) * Hkv for s in stats)},
+                           "per_beam_role": {"bytes": dec_bytes, "tokens": statistics.mean(dec_tokens)}}}
+        role = "k_attention: grouped tcgen05 role over shared segments + warp-MMA per-beam role over the tails"
     else:
-        roofline = {"bound": "hbm", "kernel": f"{dec} (split-KV decode)", "achieved": achieved, "peak": peak,
-                    "unit": "GB/s", "frac": achieved / peak,
-                    "traffic": captured_traffic(dec, wl.name, args.flags, dec_bytes), "bytes_per_launch": dec_bytes,
-                    "peak_source": f"{peak_src} hbm_gbs"}
+        kname = dec
+        k_bytes = dec_bytes
+        achieved = k_bytes / dec_avg_s / 1e9
+        kernels = {kname: {"us": dec_avg_s * 1e6, "bytes": k_bytes, "gbps": achieved, "frac_hbm": achieved / peak}}
+        role = f"{dec} (split-KV decode)"
+    roofline = {"bound": "hbm", "kernel": role, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": captured_traffic(kname, wl.name, args.flags, k_bytes),
+                "bytes_per_launch": k_bytes, "peak_source": f"{peak_src} hbm_gbs"}
 
     value = job_value(world, C, K, elapsed_ms)
     ms_per_step = elapsed_ms / K
@@ -891,8 +888,7 @@ def run_ours(args) -> None:
             "attention_us": att_avg_s * 1e6,
             "attention_tbps": eff_bytes / att_avg_s / 1e12,
             "attention_tbps_note": "every beam's whole context (K and V of all KV heads) per attention time",
-            "decode_kernel_us": dec_avg_s * 1e6,
-            "grouped_kernel_us": gr_avg_s * 1e6,
+            "attention_kernel_us": dec_avg_s * 1e6,
             "step_kernels_us": step_kernels_us,
             "probe_us": probe_us,
             "prune_branch_us": prune_us,

@@ -56,6 +56,7 @@
 // freed and the CTA leaves.
 #include <cuda.h>
 
+#include "decode_mma.cuh"
 #include "internal.cuh"
 #include "ptx.cuh"
 #include "tc.cuh"
@@ -145,26 +146,15 @@ __device__ __forceinline__ Unit load_unit(const PoolView& v, long long u) {
   return x;
 }
 
+// The grouped role of the attention kernel (k_attention, below): this CTA is one of the `ng`
+// CTAs that take grouped work units; threads past kThreads only take part in the CTA's
+// barriers.
 template <int G>
-__global__ void __launch_bounds__(kThreads, 1)
-    k_grouped(PoolView v, const __grid_constant__ CUtensorMap tm, int layer, const __nv_bfloat16* __restrict__ q,
-              float qscale, int w_oob) {
-  pdl_wait();
-  pdl_launch_dependents();
+__device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMap* tm_p, int layer,
+                                             const __nv_bfloat16* __restrict__ q, float qscale, int w_oob, int ng) {
   extern __shared__ __align__(1024) unsigned char sm[];
-  if (v.ctl[kCtlStepOk] == 0) return;
   const long long units = (long long)v.ctl[kCtlSegTiles] * v.Hkv;
   if (units == 0) return;
-  // When the per-beam kernel runs beside this one (decode_ctas), the CTAs past this
-  // kernel's share only take part in the end-of-launch ticket.
-  if ((int)blockIdx.x >= grouped_ctas(v, (int)gridDim.x)) {
-    if (threadIdx.x == 0 && atomicAdd(&v.ctl[kCtlGrpDone], 1) == (int)gridDim.x - 1) {
-      v.ctl[kCtlGrpNext] = 0;
-      v.ctl[kCtlGrpDone] = 0;
-      __threadfence();
-    }
-    return;
-  }
   if (smem_addr(sm) & 1023) {  // the swizzled layouts need a 1024-byte aligned base
     if (threadIdx.x == 0) set_status(v.ctl, GB_ERR_UNSUPPORTED);
     return;
@@ -213,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------------ K producer
-    if (lane == 0) asm volatile("prefetch.tensormap [%0];" ::"l"(&tm) : "memory");
+    if (lane == 0) asm volatile("prefetch.tensormap [%0];" ::"l"(tm_p) : "memory");
     const int ppt = kTok / v.P;                     // pages per tile (2 to 16)
     const uint32_t page_bytes = (uint32_t)v.P * 256;  // K (or V) of one page of one head
     uint32_t n = 0;  // tiles issued
@@ -296,7 +286,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         // Lane c issues page c: a TMA instruction holds its thread for a while, so the
         // lanes' copies go out in parallel.
-        if (lane < ppt) tma_page(sbase + kKRing + st * kHalfStage + lane * page_bytes, &tm, 0, w, bar);
+        if (lane < ppt) tma_page(sbase + kKRing + st * kHalfStage + lane * page_bytes, tm_p, 0, w, bar);
         if (j == 0) {
           // Query rows of the unit (after its first tile's copies are under way): row r =
           // (member, query head of this KV head); zero rows past the members.  The single
@@ -378,7 +368,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t bar = ctl + kBarVFull + 8 * st;
         if (lane == 0) mbar_arrive_expect_tx(bar, kHalfStage);
         __syncwarp();
-        if (lane < ppt) tma_page(sbase + kVRing + st * kHalfStage + lane * page_bytes, &tm, 1, w, bar);
+        if (lane < ppt) tma_page(sbase + kVRing + st * kHalfStage + lane * page_bytes, tm_p, 1, w, bar);
       }
     }
     if (lane == 0 && *abort_flag) {
@@ -504,6 +494,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     __syncwarp();
+  } else if (warp > kVProducerWarp) {
+    // threads past the grouped role's kThreads (the attention kernel's block holds the
+    // per-beam role's 12 warps): nothing to do but the CTA's barriers
   } else {
     // ------------------------------------------------------------------ softmax (warps 0-7)
     // Both groups keep the same running max per row (they swap their tile maxima through
@@ -663,12 +656,46 @@ __global__ void __launch_bounds__(kThreads, 1)
   // The last CTA to finish resets the work counter for the next launch.
   if (tid == 0) {
     __threadfence();
-    if (atomicAdd(&v.ctl[kCtlGrpDone], 1) == (int)gridDim.x - 1) {
+    if (atomicAdd(&v.ctl[kCtlGrpDone], 1) == ng - 1) {
       v.ctl[kCtlGrpNext] = 0;
       v.ctl[kCtlGrpDone] = 0;
       __threadfence();
     }
   }
+}
+
+constexpr int kAttnThreads = kMmaWarps * 32;  // the per-beam role's 12 warps; the grouped role uses 11
+static_assert(kAttnThreads >= kThreads, "the grouped role's warps fit the block");
+constexpr int kAttnSmem = kSmem > DecodeMmaSmem::TOTAL ? kSmem : DecodeMmaSmem::TOTAL;
+
+// The attention phase of a step with shared-prefix segments, in one launch of one CTA per SM:
+// the grouped role (the tcgen05 kernel above) and the per-beam role (the warp-MMA kernel of
+// decode_mma.cuh) over the step's unshared tails.  When the step reads little per SM
+// (decode_ctas), both roles are latency-bound and run side by side, each on its share of the
+// CTAs; otherwise every CTA takes grouped units until the list is exhausted and then its range
+// of the per-beam work.  Both roles write partial records that k_combine merges next.
+template <int G>
+__global__ void __launch_bounds__(kAttnThreads, 1)
+    k_attention(PoolView v, const __grid_constant__ CUtensorMap tmg, const __grid_constant__ CUtensorMap tmd,
+                const __grid_constant__ CUtensorMap tmdh, int layer, const __nv_bfloat16* __restrict__ q,
+                float qscale, int w_oob) {
+  pdl_wait();
+  pdl_launch_dependents();
+  if (v.ctl[kCtlStepOk] == 0) return;
+  const int grid = (int)gridDim.x, c = (int)blockIdx.x;
+  const int nd = decode_ctas(v, grid);  // the whole grid unless the two roles split the SMs
+  if (nd < grid) {
+    const int ng = grid - nd;
+    if (c < ng) grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, ng);
+    else decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c - ng, nd);
+    return;
+  }
+  grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, grid);
+  // The grouped role's copies and MMAs have all completed and its tensor memory is freed; the
+  // shared memory now serves the per-beam role's stages (written by the async proxy next).
+  fence_proxy_async_smem();
+  __syncthreads();
+  decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c, grid);
 }
 
 }  // namespace
@@ -721,28 +748,31 @@ void make_kv_tensor_maps(gb_pool* pool) {
 }
 
 template <int G>
-static cudaError_t launch_grouped_t(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {
+static cudaError_t launch_attention_t(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {
   {
-    const cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_grouped<G>), kSmem);
+    const cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_attention<G>), kAttnSmem);
     if (e != cudaSuccess) return e;
   }
   const PoolView& v = pool->view;
   const float qscale = scale * 1.4426950408889634f;
   prof_begin(pool, GB_PROF_GROUPED, s);
-  const cudaError_t e = launch_pdl(k_grouped<G>, pool->num_sms, kThreads, kSmem, s, v,
-                                   *reinterpret_cast<const CUtensorMap*>(pool->tmap), layer,
+  prof_begin(pool, GB_PROF_DECODE, s);
+  const cudaError_t e = launch_pdl(k_attention<G>, pool->num_sms, kAttnThreads, kAttnSmem, s, v,
+                                   *reinterpret_cast<const CUtensorMap*>(pool->tmap),
+                                   *reinterpret_cast<const CUtensorMap*>(pool->dtmap),
+                                   *reinterpret_cast<const CUtensorMap*>(pool->dtmap_half), layer,
                                    static_cast<const __nv_bfloat16*>(q), qscale, pool->tmap_oob);
+  prof_end(pool, GB_PROF_DECODE, s);
   prof_end(pool, GB_PROF_GROUPED, s);
   pool->launches += 1;
   return e;
 }
 
-cudaError_t launch_grouped(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {
-  if (!pool->view.grouped || !pool->have_tmap) return cudaSuccess;
+cudaError_t launch_attention(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {
   switch (pool->view.G) {
-    case 2: return launch_grouped_t<2>(pool, layer, q, scale, s);
-    case 4: return launch_grouped_t<4>(pool, layer, q, scale, s);
-    case 8: return launch_grouped_t<8>(pool, layer, q, scale, s);
+    case 2: return launch_attention_t<2>(pool, layer, q, scale, s);
+    case 4: return launch_attention_t<4>(pool, layer, q, scale, s);
+    case 8: return launch_attention_t<8>(pool, layer, q, scale, s);
   }
   return cudaErrorInvalidValue;
 }

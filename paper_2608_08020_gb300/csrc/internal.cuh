@@ -17,6 +17,10 @@ constexpr int kDecodeWarps = 8;    // warps per CTA of the split-KV decode kerne
 constexpr int kDecodeStages = 3;   // TMA ring depth per warp
 constexpr int kDecodeCtasPerSm = 1;
 constexpr int kMaxDecodeWarps = 4096;
+#ifndef GB_MMA_WARPS
+#define GB_MMA_WARPS 12  // warps per CTA of the warp-MMA per-beam kernel (one CTA per SM)
+#endif
+constexpr int kMmaWarps = GB_MMA_WARPS;
 constexpr int kMaxCowJobs = 1024;
 constexpr int kMaxSegDepth = 16;
 constexpr int kMaxSegRecords = 48;  // grouped partial records per beam (segments x token splits)
@@ -130,17 +134,14 @@ __host__ __device__ inline int* plan_start(const PoolView& v, int mode) {
 #define GB_SPLIT_BYTES_PER_SM (8ll << 20)
 #endif
 
-// A mode-1 step launches the grouped kernel and the per-beam kernel on two streams.
-// When the step's attention reads little per SM (below GB_SPLIT_BYTES_PER_SM), both
-// kernels are latency-bound and run side by side, each on its own share of the SMs: the
-// per-beam kernel takes decode_ctas(v, grid) of the `grid` CTAs (one per SM), in
-// proportion to its (16-token chunk x KV head) tokens against the grouped kernel's
-// (128-row tile x token) work per KV head, and the grouped kernel the rest.  Otherwise
-// each takes every CTA, and as each CTA needs most of an SM's shared memory the two run
-// one after the other.  Both kernels and the combine compute the same split from the
-// step's plan.
+// A mode-1 step launches one attention kernel with a grouped and a per-beam role.  When the
+// step's attention reads little per SM (below GB_SPLIT_BYTES_PER_SM), both roles are
+// latency-bound and run side by side, each on its own share of the CTAs (one per SM): the
+// per-beam role takes decode_ctas(v, grid) of them, in proportion to its (16-token chunk x
+// KV head) tokens against the grouped role's (128-row tile x token) work per KV head, and
+// the grouped role the rest.  Otherwise every CTA runs the grouped role and then the
+// per-beam role.  The kernel and the combine compute the same split from the step's plan.
 __device__ __forceinline__ int decode_ctas(const PoolView& v, int grid);
-__device__ __forceinline__ int grouped_ctas(const PoolView& v, int grid);
 
 // Element offset of row `row` of the K (kv=0) or V (kv=1) slab of (layer, page, head).
 __device__ __forceinline__ long long kv_elem_offset(const PoolView& v, int layer, long long page,
@@ -170,11 +171,6 @@ __device__ __forceinline__ int decode_ctas(const PoolView& v, int grid) {
   const long long wd = td * GB_DECODE_WEIGHT, wg = tg * 100;
   const long long n = (wd * grid + (wd + wg) / 2) / (wd + wg);
   return (int)(n < 1 ? 1 : (n > grid - 1 ? grid - 1 : n));
-}
-__device__ __forceinline__ int grouped_ctas(const PoolView& v, int grid) {
-  const long long td = (long long)plan_off(v, 1)[v.max_beams] * kChunk;
-  const long long tg = (long long)v.ctl[kCtlSegTileTok] * v.Hkv;
-  return split_sms(v, td, tg) ? grid - decode_ctas(v, grid) : grid;
 }
 
 __device__ __forceinline__ void set_status(int* ctl, int code) {
@@ -272,15 +268,8 @@ struct gb_pool {
   int tmap_oob = 0;                          // first row group past the tensor map (loads zeros)
   std::string last_error;
   unsigned long long launches = 0;          // kernels launched by this pool
-  cudaStream_t aux = nullptr;               // second stream: the per-beam kernel beside the grouped one
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   cudaEvent_t prof_start[GB_PROF_SLOTS] = {};  // caller-owned instrumentation events
   cudaEvent_t prof_stop[GB_PROF_SLOTS] = {};
-  ~gb_pool() {
-    if (ev_fork) cudaEventDestroy(ev_fork);
-    if (ev_join) cudaEventDestroy(ev_join);
-    if (aux) cudaStreamDestroy(aux);
-  }
 };
 
 namespace gb {
@@ -307,13 +296,14 @@ cudaError_t set_max_dynamic_smem(const void* kernel, int bytes);
 
 
 // Kernel launchers implemented in the other translation units.
-// The per-beam kernel on s_decode, then (on s, after s_decode's work) the combine.
+// The attention of one layer-step on s: mode 0, the per-beam kernel; mode 1, the attention
+// kernel with the grouped and per-beam roles (launch_attention); then the combine.
 cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
-                          cudaStream_t s, cudaStream_t s_decode);
+                          cudaStream_t s);
 cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* q, float scale, float* out,
                                cudaStream_t s);
 cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s);
-cudaError_t launch_grouped(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s);
+cudaError_t launch_attention(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s);
 void make_kv_tensor_maps(gb_pool* pool);
 cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
                          float bias, const uint8_t* mask, float* score_out, const float* scores_in,

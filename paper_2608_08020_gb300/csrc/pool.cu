@@ -553,15 +553,9 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
                   ? 1
                   : 0;
   make_kv_tensor_maps(p);
-  if (v.grouped && !p->have_tmap) v.grouped = 0;
-  // The per-beam kernel of a grouped step runs on a second stream of the pool, forked from
-  // and joined back into the caller's stream with two events.
-  if (v.grouped && (cudaStreamCreateWithFlags(&p->aux, cudaStreamNonBlocking) != cudaSuccess ||
-                    cudaEventCreateWithFlags(&p->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
-                    cudaEventCreateWithFlags(&p->ev_join, cudaEventDisableTiming) != cudaSuccess)) {
-    delete p;
-    return GB_ERR_CUDA;
-  }
+  // The grouped path runs as a role of the attention kernel beside the per-beam role, so it
+  // needs both tensor maps.
+  if (v.grouped && !(p->have_tmap && p->have_dtmap && p->num_sms * kMmaWarps <= kMaxDecodeWarps)) v.grouped = 0;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (cudaMemsetAsync(m, 0, L.partials, s) != cudaSuccess ||
       cudaMemsetAsync(m + L.seg_cover, 0, L.seg_owner - L.seg_cover, s) != cudaSuccess ||
@@ -666,18 +660,11 @@ extern "C" gb_status gb_decode_attention(gb_pool* pool, int layer, const void* q
   if (st != GB_OK) return st;
   // Mode 1: shared-prefix segments go through the grouped tensor-core kernel and the
   // per-beam kernel reads only each beam's remainder; mode 0: every beam reads everything.
-  // In mode 1 the two kernels run concurrently, each on its share of the SMs (decode_ctas):
-  // the grouped kernel on the caller's stream, the per-beam kernel on the pool's second
-  // stream, joined before the combine.
+  // In mode 1 one attention kernel runs both: the grouped and the per-beam roles on their
+  // shares of the SMs (decode_ctas), or one after the other on every SM.
   const int mode = (flags == GB_PATH_PER_BEAM || !pool->view.grouped) ? 0 : 1;
   prof_begin(pool, GB_PROF_ATTENTION, s);
-  if (mode == 1) {
-    if (cudaEventRecord(pool->ev_fork, s) != cudaSuccess || cudaStreamWaitEvent(pool->aux, pool->ev_fork, 0) != cudaSuccess)
-      return check_launch(pool, "fork");
-    if (launch_grouped(pool, layer, q_dev, scale, s) != cudaSuccess) return check_launch(pool, "grouped");
-  }
-  if (launch_decode(pool, layer, q_dev, scale, out_dev, mode, s, mode == 1 ? pool->aux : s) != cudaSuccess)
-    return check_launch(pool, "decode");
+  if (launch_decode(pool, layer, q_dev, scale, out_dev, mode, s) != cudaSuccess) return check_launch(pool, "decode");
   return check_launch(pool, "decode");
 }
 
