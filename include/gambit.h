@@ -271,14 +271,15 @@ gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_strea
  * Instrumentation (not part of the method).  Record caller-created CUDA
  * events (cudaEvent_t) immediately before and after one kernel of the
  * following calls on this pool, so a caller can time that kernel alone on its
- * own stream: `which` is GB_PROF_DECODE (the split-KV decode kernel of
- * gb_decode_attention), GB_PROF_PROBE (gb_score_probe, gb_score_mlp, or all of
- * gb_scorer_step), GB_PROF_PRUNE (all of gb_prune_branch or gb_fork_slots, the
- * shared-prefix segment rebuild included), GB_PROF_GROUPED (the grouped shared-prefix kernel),
+ * own stream: `which` is GB_PROF_DECODE (the attention launch of gb_decode_attention),
+ * GB_PROF_PROBE (gb_score_probe, gb_score_mlp, or all of gb_scorer_step), GB_PROF_PRUNE
+ * (all of gb_prune_branch or gb_fork_slots, the shared-prefix segment rebuild included),
+ * GB_PROF_GROUPED (the attention launch when it has the grouped shared-prefix role),
  * GB_PROF_PLAN (the step planner: page allocation and decode plans, layer 0),
- * GB_PROF_APPEND (the K/V append of a layer), GB_PROF_COMBINE (the merge of
- * partial results) or GB_PROF_ATTENTION (the attention kernels of a layer: the grouped
- * and per-beam kernels, which run concurrently on two streams, up to the merge).  Passing NULL events stops recording.  The events stay
+ * GB_PROF_APPEND (the K/V append of a layer), GB_PROF_COMBINE (the separate merge of
+ * partial results after the fp32 kernel; bf16 pools merge inside the attention launch) or
+ * GB_PROF_ATTENTION (the attention of a layer, up to its merged output except for the fp32
+ * kernel's separate merge).  Passing NULL events stops recording.  The events stay
  * owned by the caller.  Under stream capture the records become external event
  * nodes of the graph.
  */

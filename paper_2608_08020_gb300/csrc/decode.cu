@@ -99,11 +99,6 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
   int* s_n = s_off + (kMaxBeams + 1);
   int* s_start = s_n + (kMaxBeams + 1);
   if (v.ctl[kCtlStepOk] == 0) return;
-  if (mode == 1) {  // beside the grouped kernel: this kernel's share of the SMs (decode_ctas)
-    const int nd = decode_ctas(v, W / kDecodeWarps);
-    if ((int)blockIdx.x >= nd) return;
-    W = nd * kDecodeWarps;
-  }
   {
     const int* off = plan_off(v, mode);
     const int* nn = plan_n(v, mode);
@@ -416,26 +411,28 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 1)
 }
 
 // The per-beam kernel on its own (the per-beam path, every beam reading its whole context):
-// every CTA of the grid takes part.
+// every CTA of the grid takes part, and the pairs' records are merged into `out` in the same
+// launch (combine.cuh).
 template <int G>
 __global__ void __launch_bounds__(kMmaWarps * 32, 1)
     k_decode_mma(PoolView v, const __grid_constant__ CUtensorMap tm, const __grid_constant__ CUtensorMap tmh,
-                 int layer, const __nv_bfloat16* __restrict__ q, float qscale, int mode) {
+                 int layer, const __nv_bfloat16* __restrict__ q, float qscale, int mode, float* __restrict__ out) {
   pdl_wait();
   pdl_launch_dependents();
   decode_mma_body<G>(v, &tm, &tmh, layer, q, qscale, mode, (int)blockIdx.x, (int)gridDim.x);
+  combine_pairs<G>(v, mode, (int)gridDim.x * kMmaWarps, 0, (int)blockIdx.x, (int)gridDim.x, out);
 }
 
 // Merge the partial records of each (beam, kv head) into out[b][h*G+g][:]: the split-KV
-// records of the warps that covered the beam's per-beam range and, in mode 1, the grouped
-// records of the beam's shared-prefix segments (the log-sum-exp merge, base 2).
+// records of the warps that covered the beam's range (the log-sum-exp merge, base 2), after
+// the fp32 kernel k_decode (the bf16 kernels merge their records themselves, combine.cuh).
 // One CTA of 128 threads per (beam, kv head); thread t owns 4 consecutive output elements
 // of one query head g and folds all records in one pass, 8 records of loads in flight at a
 // time: M = running max of the records' m, acc = sum o * 2^(m - M), L = sum l * 2^(m - M),
 // rescaled when M rises.  Every thread of a warp reads the same (m, l) words (one head per
 // warp at D = 128, two at D = 64), so those loads are broadcasts; the o loads are float4
 // and coalesced.
-__global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, int wpc, float* __restrict__ out) {
+__global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, float* __restrict__ out) {
   pdl_wait();
   pdl_launch_dependents();
   const int bh = blockIdx.x;
@@ -444,23 +441,17 @@ __global__ void __launch_bounds__(128) k_combine(PoolView v, int mode, int W, in
   float* ob = out + ((size_t)b * v.Hq + (size_t)h * G) * D;
   const bool ok = v.ctl[kCtlStepOk] != 0 && v.active[b] != 0;
   const int n = ok ? plan_n(v, mode)[b] : 0;
-  const int nseg = (ok && mode == 1 && v.grouped) ? v.seg_nrec[b] : 0;  // grouped records of the beam
-  if (n == 0 && nseg == 0) {
+  if (n == 0) {
     for (int e = threadIdx.x; e < GD; e += blockDim.x) ob[e] = 0.f;
     return;
   }
   const int Tot = plan_off(v, mode)[v.max_beams];
-  if (mode == 1) W = decode_ctas(v, W / wpc) * wpc;  // the warps the decode kernel used (wpc per CTA)
   const int c = Tot > 0 ? (Tot + W - 1) / W : 1;
   const int off = plan_off(v, mode)[b] + h * n;
   const int first = off / c, npb = n > 0 ? (off + n - 1) / c - first + 1 : 0;  // per-beam records
-  const int R = npb + nseg;
+  const int R = npb;
   const float* prec = v.partials + (size_t)(first + bh) * v.record_floats;
-  const float* grec = v.grec + ((size_t)b * kMaxSegRecords * v.Hkv + h) * v.record_floats;
-  const size_t gstride = (size_t)v.Hkv * v.record_floats;
-  auto rec_at = [&](int r) -> const float* {
-    return r < npb ? prec + (size_t)r * v.record_floats : grec + (size_t)(r - npb) * gstride;
-  };
+  auto rec_at = [&](int r) -> const float* { return prec + (size_t)r * v.record_floats; };
   const bool vec_out = (reinterpret_cast<uintptr_t>(ob) & 15) == 0;
   for (int e4 = threadIdx.x; e4 < GD / 4; e4 += blockDim.x) {
     const int g = (e4 * 4) / D;
@@ -522,15 +513,12 @@ template <int DT, int G>
 static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
                                    cudaStream_t s) {
   using S = DecodeSmem<DT, G>;
-  int W = pool->decode_warps, wpc = kDecodeWarps;  // warps launched, warps per CTA (one CTA per SM)
   const float qscale = scale * 1.4426950408889634f;  // log2(e): softmax in base 2
   cudaError_t e;
   if (DT == GB_BF16 && pool->have_dtmap && pool->num_sms * kMmaWarps <= kMaxDecodeWarps) {
-    wpc = kMmaWarps;
-    W = pool->num_sms * kMmaWarps;  // one CTA per SM
+    // One launch: the attention roles and the merge of their records.
     if (mode == 1) {
-      // The grouped and per-beam roles in one launch (grouped.cu).
-      e = launch_attention(pool, layer, q, scale, s);
+      e = launch_attention(pool, layer, q, scale, out, s);  // grouped and per-beam roles (grouped.cu)
     } else {
       e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_decode_mma<G>), DecodeMmaSmem::TOTAL);
       if (e != cudaSuccess) return e;
@@ -538,24 +526,26 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
       e = launch_pdl(k_decode_mma<G>, pool->num_sms, kMmaWarps * 32, DecodeMmaSmem::TOTAL, s, pool->view,
                      *reinterpret_cast<const CUtensorMap*>(pool->dtmap),
                      *reinterpret_cast<const CUtensorMap*>(pool->dtmap_half), layer,
-                     static_cast<const __nv_bfloat16*>(q), qscale, mode);
+                     static_cast<const __nv_bfloat16*>(q), qscale, mode, out);
       prof_end(pool, GB_PROF_DECODE, s);
       pool->launches += 1;
     }
-  } else {
-    if (mode == 1) return cudaErrorInvalidValue;  // a grouped pool always has the per-beam tensor maps
-    e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_decode<DT, G>), S::TOTAL);
-    if (e != cudaSuccess) return e;
-    prof_begin(pool, GB_PROF_DECODE, s);
-    e = launch_pdl(k_decode<DT, G>, W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s, pool->view, layer, q, qscale,
-                   mode, W);
-    prof_end(pool, GB_PROF_DECODE, s);
-    pool->launches += 1;
+    prof_end(pool, GB_PROF_ATTENTION, s);
+    return e;
   }
+  if (mode == 1) return cudaErrorInvalidValue;  // a grouped pool always has the per-beam tensor maps
+  const int W = pool->decode_warps;  // one CTA of kDecodeWarps warps per SM
+  e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_decode<DT, G>), S::TOTAL);
+  if (e != cudaSuccess) return e;
+  prof_begin(pool, GB_PROF_DECODE, s);
+  e = launch_pdl(k_decode<DT, G>, W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s, pool->view, layer, q, qscale,
+                 mode, W);
+  prof_end(pool, GB_PROF_DECODE, s);
+  pool->launches += 1;
   if (e != cudaSuccess) return e;
   prof_end(pool, GB_PROF_ATTENTION, s);
   prof_begin(pool, GB_PROF_COMBINE, s);
-  e = launch_pdl(k_combine, pool->view.max_beams * pool->view.Hkv, 128, 0, s, pool->view, mode, W, wpc, out);
+  e = launch_pdl(k_combine, pool->view.max_beams * pool->view.Hkv, 128, 0, s, pool->view, mode, W, out);
   prof_end(pool, GB_PROF_COMBINE, s);
   pool->launches += 1;
   return e;
@@ -575,7 +565,7 @@ static cudaError_t launch_view_t(const PoolView& v, int W, int layer, const void
   k_decode<DT, G><<<W / kDecodeWarps, kDecodeWarps * 32, S::TOTAL, s>>>(v, layer, q, qscale, 0, W);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_combine<<<v.max_beams * v.Hkv, 128, 0, s>>>(v, 0, W, kDecodeWarps, out);
+  k_combine<<<v.max_beams * v.Hkv, 128, 0, s>>>(v, 0, W, out);
   return cudaGetLastError();
 }
 

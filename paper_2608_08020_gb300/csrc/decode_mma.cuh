@@ -6,6 +6,7 @@
 #include <cuda_bf16.h>
 #include <math.h>
 
+#include "combine.cuh"
 #include "internal.cuh"
 #include "ptx.cuh"
 
@@ -375,6 +376,7 @@ __device__ __forceinline__ void decode_mma_body(const PoolView& v, const CUtenso
           rec[G * D + G + 2 * c + 1] = l1;
         }
       }
+      record_arrive(v, it.b * v.Hkv + it.h, lane);
       fresh = true;
     }
     if (x + 1 < x_end) iter_advance(it, s_n, s_start, v.Hkv, v.max_beams);

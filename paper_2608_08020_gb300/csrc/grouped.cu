@@ -653,15 +653,6 @@ __device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMa
   __syncthreads();
   tc_fence_after();
   if (warp == kMmaWarp) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
-  // The last CTA to finish resets the work counter for the next launch.
-  if (tid == 0) {
-    __threadfence();
-    if (atomicAdd(&v.ctl[kCtlGrpDone], 1) == ng - 1) {
-      v.ctl[kCtlGrpNext] = 0;
-      v.ctl[kCtlGrpDone] = 0;
-      __threadfence();
-    }
-  }
 }
 
 constexpr int kAttnThreads = kMmaWarps * 32;  // the per-beam role's 12 warps; the grouped role uses 11
@@ -673,29 +664,38 @@ constexpr int kAttnSmem = kSmem > DecodeMmaSmem::TOTAL ? kSmem : DecodeMmaSmem::
 // decode_mma.cuh) over the step's unshared tails.  When the step reads little per SM
 // (decode_ctas), both roles are latency-bound and run side by side, each on its share of the
 // CTAs; otherwise every CTA takes grouped units until the list is exhausted and then its range
-// of the per-beam work.  Both roles write partial records that k_combine merges next.
+// of the per-beam work.  The pairs' records are merged into `out` in the same launch
+// (combine.cuh).
 template <int G>
 __global__ void __launch_bounds__(kAttnThreads, 1)
     k_attention(PoolView v, const __grid_constant__ CUtensorMap tmg, const __grid_constant__ CUtensorMap tmd,
                 const __grid_constant__ CUtensorMap tmdh, int layer, const __nv_bfloat16* __restrict__ q,
-                float qscale, int w_oob) {
+                float qscale, int w_oob, float* __restrict__ out) {
   pdl_wait();
   pdl_launch_dependents();
-  if (v.ctl[kCtlStepOk] == 0) return;
   const int grid = (int)gridDim.x, c = (int)blockIdx.x;
-  const int nd = decode_ctas(v, grid);  // the whole grid unless the two roles split the SMs
-  if (nd < grid) {
-    const int ng = grid - nd;
-    if (c < ng) grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, ng);
-    else decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c - ng, nd);
-    return;
+  int nd = grid, ng = grid;  // CTAs of the per-beam and the grouped role
+  if (v.ctl[kCtlStepOk] != 0) {
+    nd = decode_ctas(v, grid);  // the whole grid unless the two roles split the SMs
+    if (nd < grid) {
+      ng = grid - nd;
+      if (c < ng) {
+        grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, ng);
+        grouped_cta_done(v);
+      } else {
+        decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c - ng, nd);
+      }
+    } else {
+      grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, grid);
+      grouped_cta_done(v);
+      // The grouped role's copies and MMAs have all completed and its tensor memory is freed;
+      // the shared memory now serves the per-beam role's stages (written by the async proxy).
+      fence_proxy_async_smem();
+      __syncthreads();
+      decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c, grid);
+    }
   }
-  grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, grid);
-  // The grouped role's copies and MMAs have all completed and its tensor memory is freed; the
-  // shared memory now serves the per-beam role's stages (written by the async proxy next).
-  fence_proxy_async_smem();
-  __syncthreads();
-  decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c, grid);
+  combine_pairs<G>(v, 1, nd * kMmaWarps, ng, c, grid, out);
 }
 
 }  // namespace
@@ -748,7 +748,8 @@ void make_kv_tensor_maps(gb_pool* pool) {
 }
 
 template <int G>
-static cudaError_t launch_attention_t(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {
+static cudaError_t launch_attention_t(gb_pool* pool, int layer, const void* q, float scale, float* out,
+                                      cudaStream_t s) {
   {
     const cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_attention<G>), kAttnSmem);
     if (e != cudaSuccess) return e;
@@ -761,18 +762,18 @@ static cudaError_t launch_attention_t(gb_pool* pool, int layer, const void* q, f
                                    *reinterpret_cast<const CUtensorMap*>(pool->tmap),
                                    *reinterpret_cast<const CUtensorMap*>(pool->dtmap),
                                    *reinterpret_cast<const CUtensorMap*>(pool->dtmap_half), layer,
-                                   static_cast<const __nv_bfloat16*>(q), qscale, pool->tmap_oob);
+                                   static_cast<const __nv_bfloat16*>(q), qscale, pool->tmap_oob, out);
   prof_end(pool, GB_PROF_DECODE, s);
   prof_end(pool, GB_PROF_GROUPED, s);
   pool->launches += 1;
   return e;
 }
 
-cudaError_t launch_attention(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s) {
+cudaError_t launch_attention(gb_pool* pool, int layer, const void* q, float scale, float* out, cudaStream_t s) {
   switch (pool->view.G) {
-    case 2: return launch_attention_t<2>(pool, layer, q, scale, s);
-    case 4: return launch_attention_t<4>(pool, layer, q, scale, s);
-    case 8: return launch_attention_t<8>(pool, layer, q, scale, s);
+    case 2: return launch_attention_t<2>(pool, layer, q, scale, out, s);
+    case 4: return launch_attention_t<4>(pool, layer, q, scale, out, s);
+    case 8: return launch_attention_t<8>(pool, layer, q, scale, out, s);
   }
   return cudaErrorInvalidValue;
 }

@@ -44,8 +44,8 @@ enum Ctl : int {
   kCtlSegTileTok = 11, // sum over segments of (128-row tiles) x tokens
   kCtlSteps = 12,      // steps opened so far (index into the step-stats ring)
   kCtlSegSplit = 13,   // tokens per grouped work unit (segments are split along tokens)
-  kCtlGrpNext = 14,    // next grouped work unit to hand out (reset by the grouped kernel's last CTA)
-  kCtlGrpDone = 15,    // grouped-kernel CTAs finished (reset by the last one)
+  kCtlGrpNext = 14,    // next grouped work unit to hand out (zeroed by k_append)
+  kCtlGrpDone = 15,    // grouped-role CTAs finished (zeroed by k_append)
   kCtlSegTok = 16,     // sum over segments of their tokens (the shared tokens the grouped path reads once)
   kCtlBarCount = 17,   // grid-barrier arrivals of the tournament kernel (only grows)
   kCtlSegGen = 19,     // segment rebuilds so far (stamps the per-page claim words)
@@ -59,7 +59,7 @@ struct MetaLayout {
   size_t plan, cow, partials, total, stats;
   // shared-prefix segments
   size_t seg_cover, seg_nseg, seg_owner, seg_i0, seg_len, seg_rep, seg_g, seg_mem_off, seg_fill, seg_members,
-      seg_tile_seg, seg_tile_t, grec, seg_bid, seg_rec_off, seg_nrec, seg_splits, seg_tile_split, seg_hist;
+      seg_tile_seg, seg_tile_t, grec, seg_bid, seg_rec_off, seg_nrec, seg_splits, seg_tile_split, seg_hist, pair_cnt;
   int words;            // free-bitmap words
   size_t mlp_scratch;   // MLP scorer partial sums
   int partial_records;  // split-KV partial records
@@ -111,6 +111,8 @@ struct PoolView {
   float* grec;          // [max_beams][kMaxSegDepth][Hkv] grouped partial records
   int* stats;           // [kStatsRing][kStatsWords] work of recent steps (see gb_pool_read_step_stats)
   float* partials;
+  int* pair_cnt;        // [max_beams * Hkv] per-beam records written for each (beam, KV head) by the
+                        // running attention launch (zeroed by k_append before it)
   int record_floats;
   float* mlp_scratch;   // [kMlpScratchFloats] K-split partials of the MLP scorer
 };
@@ -127,7 +129,7 @@ __host__ __device__ inline int* plan_start(const PoolView& v, int mode) {
 }
 
 #ifndef GB_DECODE_WEIGHT
-#define GB_DECODE_WEIGHT 60  // relative cost of a per-beam token against a grouped tile token (percent)
+#define GB_DECODE_WEIGHT 45  // relative cost of a per-beam token against a grouped tile token (percent)
 #endif
 
 #ifndef GB_SPLIT_BYTES_PER_SM
@@ -296,14 +298,15 @@ cudaError_t set_max_dynamic_smem(const void* kernel, int bytes);
 
 
 // Kernel launchers implemented in the other translation units.
-// The attention of one layer-step on s: mode 0, the per-beam kernel; mode 1, the attention
-// kernel with the grouped and per-beam roles (launch_attention); then the combine.
+// The attention of one layer-step on s, written to out: mode 0, the per-beam kernel; mode 1,
+// the attention kernel with the grouped and per-beam roles (launch_attention).  The bf16
+// kernels merge their records themselves; the fp32 kernel is followed by k_combine.
 cudaError_t launch_decode(gb_pool* pool, int layer, const void* q, float scale, float* out, int mode,
                           cudaStream_t s);
 cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* q, float scale, float* out,
                                cudaStream_t s);
 cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s);
-cudaError_t launch_attention(gb_pool* pool, int layer, const void* q, float scale, cudaStream_t s);
+cudaError_t launch_attention(gb_pool* pool, int layer, const void* q, float scale, float* out, cudaStream_t s);
 void make_kv_tensor_maps(gb_pool* pool);
 cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
                          float bias, const uint8_t* mask, float* score_out, const float* scores_in,

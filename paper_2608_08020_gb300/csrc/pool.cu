@@ -39,7 +39,7 @@ MetaLayout meta_layout(const gb_pool_config& c) {
   m.plan = take(2 * 3 * (B + 1) * sizeof(int));
   m.cow = take(kMaxCowJobs * 3 * sizeof(int));
   m.record_floats = G * (c.head_dim + 2);
-  m.partial_records = kMaxDecodeWarps + (int)B * c.num_kv_heads;
+  m.partial_records = kMaxDecodeWarps + (int)B * c.num_kv_heads;  // record index: warp + b * Hkv + h
   m.partials = take((size_t)m.partial_records * m.record_floats * sizeof(float));
   const size_t BD = B * kMaxSegDepth;
   m.seg_cover = take(B * sizeof(int));
@@ -61,6 +61,7 @@ MetaLayout meta_layout(const gb_pool_config& c) {
   m.seg_splits = take(BD * sizeof(int));
   m.seg_tile_split = take(B * kMaxSegRecords * sizeof(int));
   m.seg_hist = take(2 * 256 * sizeof(int));
+  m.pair_cnt = take(B * c.num_kv_heads * sizeof(int));
   m.stats = take((size_t)kStatsRing * kStatsWords * sizeof(int));
   m.mlp_scratch = take((size_t)kMlpScratchFloats * sizeof(float));
   m.total = o;
@@ -357,6 +358,15 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
 __global__ void k_append(PoolView v, int layer, int n_tokens, const char* kin, const char* vin) {
   pdl_wait();
   pdl_launch_dependents();
+  // The counters of the attention launch that follows (combine.cuh, the grouped role's
+  // work queue): the previous attention launch has completed (pdl_wait).
+  if (blockIdx.x == 0 && blockIdx.y == 0) {
+    for (int i = threadIdx.x; i < v.max_beams * v.Hkv; i += blockDim.x) v.pair_cnt[i] = 0;
+    if (threadIdx.x == 0) {
+      v.ctl[kCtlGrpNext] = 0;
+      v.ctl[kCtlGrpDone] = 0;
+    }
+  }
   if (v.ctl[kCtlStepOk] == 0) return;
   const int vec_per_row = v.D * v.esize / 16;
   // Copy-on-write of still-shared partial tail pages, this layer's rows [0, rows).
@@ -542,6 +552,7 @@ extern "C" gb_status gb_pool_init(const gb_pool_config* cfg, void* kv_dev, void*
   v.seg_splits = reinterpret_cast<int*>(m + L.seg_splits);
   v.seg_tile_split = reinterpret_cast<int*>(m + L.seg_tile_split);
   v.seg_hist = reinterpret_cast<int*>(m + L.seg_hist);
+  v.pair_cnt = reinterpret_cast<int*>(m + L.pair_cnt);
   v.num_sms = p->num_sms;
   v.stats = reinterpret_cast<int*>(m + L.stats);
   v.mlp_scratch = reinterpret_cast<float*>(m + L.mlp_scratch);

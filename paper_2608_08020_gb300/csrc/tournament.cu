@@ -74,7 +74,6 @@ __device__ __forceinline__ void unref_page_cta(const PoolView& v, int p, int* s_
   }
 }
 
-__device__ __forceinline__ void fence_acq_rel_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 
 // Grid-wide barrier over a grid whose CTAs are all resident.  The arrival counter only ever
 // grows: barrier n of a grid of G CTAs is passed once it reaches the next multiple of G above
