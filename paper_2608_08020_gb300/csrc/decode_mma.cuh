@@ -381,6 +381,9 @@ __device__ __forceinline__ void decode_mma_body(const PoolView& v, const CUtenso
     }
     if (x + 1 < x_end) iter_advance(it, s_n, s_start, v.Hkv, v.max_beams);
   }
+  // Every chunk this warp issued has been consumed: its barriers' memory may serve again.
+  if (lane == 0)
+    for (int s = 0; s < kMmaStages; ++s) mbar_inval(bar0 + 8 * s);
 }
 
 

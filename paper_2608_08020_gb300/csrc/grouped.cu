@@ -9,7 +9,7 @@
 // split); a persistent grid of one CTA per SM walks the flat unit list, and the tiles of
 // all of a CTA's units form one continuous pipeline.
 //
-// Warp roles (352 threads):
+// Warp roles (352 of the attention kernel's 384 threads; the last warp idles in this role):
 //   warps 0-3  softmax group 0 and warps 4-7 softmax group 1: thread r of group k owns
 //              query row r (TMEM lane r) and tokens [64k, 64k + 64) of every tile.  Each
 //              tile the two groups swap their row maxima through shared memory, so both
@@ -31,8 +31,8 @@
 //              P.V takes P straight from tensor memory.
 // Handshakes are mbarriers: full/empty per K stage and per V stage, sched_full/sched_empty
 // per unit slot, q_full/q_empty, s_full, p_full and pv_done per S/P tile (three in
-// tensor memory), max_full per tile parity, xch_full and o_free per unit.  The last CTA
-// to finish resets the grid-wide counters.  An S/P buffer is reused by S(n+3) only after
+// tensor memory), max_full per tile parity, xch_full and o_free per unit.  The grid-wide
+// work counter is zeroed by k_append before each launch.  An S/P buffer is reused by S(n+3) only after
 // P.V(n) has been issued: the tensor core runs a CTA's MMAs in issue order, so P(n) has
 // been read before S(n+3) overwrites it.  With three buffers S runs two tiles ahead of
 // the softmax.
@@ -653,6 +653,9 @@ __device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMa
   __syncthreads();
   tc_fence_after();
   if (warp == kMmaWarp) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
+  // Every copy and MMA has completed: the barriers' memory may serve the per-beam role next.
+  if (tid == 0)
+    for (int b = 0; b < kWordSched; b += 8) mbar_inval(ctl + b);
 }
 
 constexpr int kAttnThreads = kMmaWarps * 32;  // the per-beam role's 12 warps; the grouped role uses 11

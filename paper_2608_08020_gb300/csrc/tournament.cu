@@ -172,34 +172,40 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
     childof[tid] = -1;
     int N;
     const int pos = block_exclusive_scan(act ? 1 : 0, tmp, &N);
-    int npow = 1;
-    while (npow < N) npow <<= 1;
     s_keys[tid] = ~0ull;
     __syncthreads();
     if (act) s_keys[pos] = ((unsigned long long)rank_key(v.mean[tid]) << 32) | (unsigned)tid;
     __syncthreads();
-    // Bitonic sort of the first npow keys, ascending, by the warps that hold them: strides
-    // >= 32 through shared memory (a named barrier over those warps), strides < 32 by
-    // shuffles inside a warp.  Threads >= npow of those warps only meet each other.
-    const int sort_threads = npow < 32 ? 32 : npow;
-    if (tid < sort_threads) {
-      unsigned long long my = s_keys[tid];
-      for (int k = 2; k <= npow; k <<= 1) {
+    // Rank (ascending keys; the slot in the low word makes them distinct): each warp sorts its
+    // 32 keys in registers (bitonic, by shuffles), then a key's rank is its position in its
+    // warp's list plus, for every other list, the number of keys there below it (a binary
+    // search over 32 sorted keys; four lists at a time).
+    const int nl = (N + 31) >> 5, lane = tid & 31, wl = tid >> 5;
+    if (wl < nl) {
+      unsigned long long my = s_keys[tid];  // ~0 past the N keys
+      for (int k = 2; k <= 32; k <<= 1)
         for (int j = k >> 1; j > 0; j >>= 1) {
-          unsigned long long other;
-          if (j >= 32) {
-            asm volatile("bar.sync 1, %0;" ::"r"(sort_threads) : "memory");
-            s_keys[tid] = my;
-            asm volatile("bar.sync 1, %0;" ::"r"(sort_threads) : "memory");
-            other = s_keys[tid ^ j];
-          } else {
-            other = __shfl_xor_sync(0xffffffffu, my, j);
-          }
-          const bool asc = (tid & k) == 0, lower = (tid & j) == 0;
+          const unsigned long long other = __shfl_xor_sync(0xffffffffu, my, j);
+          const bool asc = (lane & k) == 0, lower = (lane & j) == 0;
           my = (asc == lower) ? (my < other ? my : other) : (my > other ? my : other);
         }
+      s_keys[tid] = my;
+      asm volatile("bar.sync 1, %0;" ::"r"(nl * 32) : "memory");
+      if (my != ~0ull) {
+        int rank = lane;
+        for (int l0 = 0; l0 < nl; l0 += 4) {
+          int pos[4] = {0, 0, 0, 0};
+#pragma unroll
+          for (int st = 16; st > 0; st >>= 1)
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+              if (l0 + u < nl && s_keys[32 * (l0 + u) + pos[u] + st - 1] < my) pos[u] += st;
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+            if (l0 + u < nl && l0 + u != wl) rank += pos[u] + (s_keys[32 * (l0 + u) + pos[u]] < my ? 1 : 0);
+        }
+        ord[rank] = (int)(my & 0xffffffffu);
       }
-      if (tid < N) ord[tid] = (int)(my & 0xffffffffu);
     }
     __syncthreads();
     // Routing (identical in every CTA).
