@@ -32,10 +32,10 @@
 // Handshakes are mbarriers: full/empty per K stage and per V stage, sched_full/sched_empty
 // per unit slot, q_full/q_empty, s_full, p_full and pv_done per S/P tile (three in
 // tensor memory), max_full per tile parity, xch_full and o_free per unit.  The grid-wide
-// work counter is zeroed by k_append before each launch.  An S/P buffer is reused by S(n+3) only after
-// P.V(n) has been issued: the tensor core runs a CTA's MMAs in issue order, so P(n) has
-// been read before S(n+3) overwrites it.  With three buffers S runs two tiles ahead of
-// the softmax.
+// work counter is zeroed by k_append before each launch.  An S/P buffer is reused by
+// S(n+3) only after P.V(n) has been issued: the tensor core runs a CTA's MMAs in issue
+// order, so P(n) has been read before S(n+3) overwrites it.  With three buffers S runs two
+// tiles ahead of the softmax.
 //
 // Shared memory (dynamic only, 1024-byte aligned, 128-byte swizzle everywhere):
 //   Q     two [128 rows][64 dims] blocks (K-major A operand)                32 KiB
