@@ -662,13 +662,12 @@ constexpr int kAttnThreads = kMmaWarps * 32;  // the per-beam role's 12 warps; t
 static_assert(kAttnThreads >= kThreads, "the grouped role's warps fit the block");
 constexpr int kAttnSmem = kSmem > DecodeMmaSmem::TOTAL ? kSmem : DecodeMmaSmem::TOTAL;
 
-// The attention phase of a step with shared-prefix segments, in one launch of one CTA per SM:
-// the grouped role (the tcgen05 kernel above) and the per-beam role (the warp-MMA kernel of
-// decode_mma.cuh) over the step's unshared tails.  When the step reads little per SM
+// The attention phase of a step with shared-prefix segments, in one launch: the grouped role
+// (the tcgen05 kernel above) and the per-beam role (the warp-MMA kernel of decode_mma.cuh)
+// over the step's unshared tails, one CTA per SM at a time.  When the step reads little per SM
 // (decode_ctas), both roles are latency-bound and run side by side, each on its share of the
-// CTAs; otherwise every CTA takes grouped units until the list is exhausted and then its range
-// of the per-beam work.  The pairs' records are merged into `out` in the same launch
-// (combine.cuh).
+// SMs; otherwise the per-beam CTAs follow the grouped ones onto the SMs they leave.  The
+// pairs' records are merged into `out` in the same launch (combine.cuh).
 template <int G>
 __global__ void __launch_bounds__(kAttnThreads, 1)
     k_attention(PoolView v, const __grid_constant__ CUtensorMap tmg, const __grid_constant__ CUtensorMap tmd,
@@ -676,29 +675,32 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 float qscale, int w_oob, float* __restrict__ out) {
   pdl_wait();
   pdl_launch_dependents();
-  const int grid = (int)gridDim.x, c = (int)blockIdx.x;
-  int nd = grid, ng = grid;  // CTAs of the per-beam and the grouped role
-  if (v.ctl[kCtlStepOk] != 0) {
-    nd = decode_ctas(v, grid);  // the whole grid unless the two roles split the SMs
-    if (nd < grid) {
-      ng = grid - nd;
-      if (c < ng) {
-        grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, ng);
-        grouped_cta_done(v);
-      } else {
-        decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c - ng, nd);
-      }
-    } else {
-      grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, grid);
-      grouped_cta_done(v);
-      // The grouped role's copies and MMAs have all completed and its tensor memory is freed;
-      // the shared memory now serves the per-beam role's stages (written by the async proxy).
-      fence_proxy_async_smem();
-      __syncthreads();
-      decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c, grid);
-    }
+  // Grid of 2 S CTAs (S = SM count).  Large steps: CTAs [0, S) take the grouped role and
+  // leave, CTAs [S, 2S) the per-beam role, each on an SM as a grouped CTA leaves it (CTAs
+  // start in index order), and merge the records; a grouped CTA never waits, so every
+  // per-beam CTA gets an SM.  Small steps: [0, ng) grouped and [ng, S) per-beam side by side,
+  // all S resident at once, all S merging; the rest leave at once.
+  const int S = (int)gridDim.x / 2, c = (int)blockIdx.x;
+  const bool ok = v.ctl[kCtlStepOk] != 0;
+  int nd = S, ng = S;
+  if (ok) {
+    nd = decode_ctas(v, S);
+    if (nd < S) ng = S - nd;
   }
-  combine_pairs<G>(v, 1, nd * kMmaWarps, ng, c, grid, out);
+  const bool split = nd < S;
+  const int pb0 = split ? ng : S;  // first per-beam CTA
+  if (c >= pb0 + nd) return;
+  if (c < pb0) {
+    if (ok) {
+      grouped_body<G>(v, &tmg, layer, q, qscale, w_oob, ng);
+      grouped_cta_done(v);
+    }
+    if (!split) return;
+  } else {
+    decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c - pb0, nd);
+  }
+  if (split) combine_pairs<G>(v, 1, nd * kMmaWarps, ng, c, S, out);
+  else combine_pairs<G>(v, 1, nd * kMmaWarps, ng, c - S, S, out);
 }
 
 }  // namespace
@@ -761,7 +763,7 @@ static cudaError_t launch_attention_t(gb_pool* pool, int layer, const void* q, f
   const float qscale = scale * 1.4426950408889634f;
   prof_begin(pool, GB_PROF_GROUPED, s);
   prof_begin(pool, GB_PROF_DECODE, s);
-  const cudaError_t e = launch_pdl(k_attention<G>, pool->num_sms, kAttnThreads, kAttnSmem, s, v,
+  const cudaError_t e = launch_pdl(k_attention<G>, 2 * pool->num_sms, kAttnThreads, kAttnSmem, s, v,
                                    *reinterpret_cast<const CUtensorMap*>(pool->tmap),
                                    *reinterpret_cast<const CUtensorMap*>(pool->dtmap),
                                    *reinterpret_cast<const CUtensorMap*>(pool->dtmap_half), layer,
