@@ -28,10 +28,25 @@ pytestmark = pytest.mark.gpu
 @pytest.mark.parametrize("config,path", [(2, "auto"), (2, "per_beam"), (3, "auto"), (4, "auto"), (5, "auto"),
                                          (6, "auto"), (6, "per_beam")])
 def test_full_size_sampled_beams_match_oracle(cuda, config, path):
+    _check_full_size(BY_INDEX[config - 1], path)
+
+
+# Query heads per KV head G = 2 and 8 on the 64-beam tree (the attention launch's two roles side
+# by side on their shares of the SMs) and on the 512-beam tree (the per-beam CTAs following the
+# grouped ones: 2-4 GB of attention reads per step).
+@pytest.mark.parametrize("config,hq,hkv", [(2, 16, 8), (2, 32, 4), (3, 16, 8), (3, 32, 4)])
+def test_full_size_group_sizes_match_oracle(cuda, config, hq, hkv):
+    import dataclasses
+
+    base = BY_INDEX[config - 1]
+    _check_full_size(dataclasses.replace(base, name=f"{base.name}-G{hq // hkv}", num_q_heads=hq, num_kv_heads=hkv),
+                     "auto")
+
+
+def _check_full_size(wl, path):
     import torch
 
     from workload.driver import GpuRun
-    wl = BY_INDEX[config - 1]
     max_context = wl.context + 1                      # bench.py's pool sizing (every phase ends at the context)
     g = GpuRun(wl, device_gen=True, max_context=max_context)
     o = OracleRun(wl, literal_kv=False, max_context=max_context)
