@@ -141,8 +141,15 @@ gb_status gb_pool_seed(gb_pool* pool, int n_beams, int prompt_len, const void* k
  *   out_dev:    [max_beams][Hq][D] fp32 (rows of inactive slots are zero)
  *   flags:      GB_PATH_AUTO / GB_PATH_PER_BEAM / GB_PATH_GROUPED
  * Rows of inactive slots in the inputs are ignored.
+ * Launches: the append, then one attention launch that also merges the
+ * split and shared-prefix partial results into out_dev (bf16 pools; fp32
+ * pools add a merge launch); layer 0 adds the step's planner first.  The
+ * attention launch's CTAs wait (bounded) on each other's partial results, so
+ * they must all get an SM within the wait limit (2 s): nothing else should
+ * hold the GPU's SMs for that long meanwhile.
  * Errors: GB_ERR_STATE for a layer out of order; out of pages is reported in
- * the device status and makes the whole step a no-op.
+ * the device status and makes the whole step a no-op; a wait that runs out
+ * records GB_ERR_TIMEOUT and zeroes the outputs it could not complete.
  */
 gb_status gb_decode_attention(gb_pool* pool, int layer, const void* q_dev, const void* k_new_dev,
                               const void* v_new_dev, float scale, float* out_dev, int flags,
