@@ -63,18 +63,6 @@ __device__ __forceinline__ unsigned rank_key(float m) {
   return ~asc;
 }
 
-// Drop one reference to page p; a page reaching zero is marked free in the bitmap, and the
-// CTA's count of freed pages and lowest freed bitmap word are kept in shared memory (added to
-// the pool's counters once per CTA instead of once per page).
-__device__ __forceinline__ void unref_page_cta(const PoolView& v, int p, int* s_freed, int* s_minword) {
-  if (atomicSub(&v.refcnt[p], 1) == 1) {
-    atomicOr(&v.free_bits[p >> 5], 1u << (p & 31));
-    atomicMin(s_minword, p >> 5);
-    atomicAdd(s_freed, 1);
-  }
-}
-
-
 // Grid-wide barrier over a grid whose CTAs are all resident.  The arrival counter only ever
 // grows: barrier n of a grid of G CTAs is passed once it reaches the next multiple of G above
 // a CTA's own arrival, so the last arrival releases everyone with no reset (the count is a
@@ -126,6 +114,7 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
   __shared__ int blist[kMaxBeams];    // eligible parents in rank order
   __shared__ int cslot[kMaxBeams];    // child k -> slot
   __shared__ int childof[kMaxBeams];  // slot -> child index or -1
+  __shared__ int s_oldn[kMaxBeams];   // child k -> table entries its slot held before the fork
   __shared__ unsigned char s_act[kMaxBeams], s_elig[kMaxBeams], s_pruned[kMaxBeams];
   __shared__ int s_pref[kTourThreads];
   __shared__ int tmp[33];
@@ -260,7 +249,15 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
     // Fork: this CTA's parents, each by its own group of threads (ppc parents at a time).  For
     // table index i of parent p, each child c either already holds page tp[i] (nothing
     // changes) or drops its old page and takes tp[i]; the new references of one parent's page
-    // are added at once.
+    // are added at once.  A page whose last reference drops is marked free in the bitmap; the
+    // CTA's count of freed pages and lowest freed bitmap word are kept in shared memory and
+    // added to the pool's counters once per CTA.
+    // The children's table lengths before the fork, one load per child for all its entries.
+    for (int c = tid; c < nchild; c += blockDim.x) {
+      const int sl = cslot[c];
+      s_oldn[c] = s_act[sl] ? (v.seq_len[sl] + v.P - 1) / v.P : 0;
+    }
+    __syncthreads();
     const int mine = npar > (int)blockIdx.x ? (npar - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
     int ppc = 1;
     while (ppc < 32 && ppc < mine) ppc <<= 1;
@@ -270,23 +267,34 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
       const int k0 = j * per, k1 = min(k0 + per, nchild);
       const int new_n = (v.seq_len[p] + v.P - 1) / v.P;
       int m = new_n;
-      for (int c = k0; c < k1; ++c) {
-        const int sl = cslot[c];
-        m = max(m, s_act[sl] ? (v.seq_len[sl] + v.P - 1) / v.P : 0);
-      }
+      for (int c = k0; c < k1; ++c) m = max(m, s_oldn[c]);
       const int* tp = v.tables + (size_t)p * v.max_pages;
       for (int i = ft; i < m; i += tpp) {
         const int nw = i < new_n ? tp[i] : -1;
         int add = 0;
-        for (int c = k0; c < k1; ++c) {
-          const int sl = cslot[c];
-          const int old_n = s_act[sl] ? (v.seq_len[sl] + v.P - 1) / v.P : 0;
-          int* ts = v.tables + (size_t)sl * v.max_pages;
-          const int old = i < old_n ? ts[i] : -1;
-          if (old == nw) continue;
-          if (nw >= 0) ++add;
-          if (old >= 0) unref_page_cta(v, old, &s_freed, &s_minword);
-          if (i < new_n) ts[i] = nw;
+        // Four children at a time: their old entries, then their reference drops, are
+        // issued together rather than one child after another.
+        for (int c0 = k0; c0 < k1; c0 += 4) {
+          int old[4], dec[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int c = c0 + u;
+            old[u] = nw;  // no child: nothing changes
+            if (c < k1) old[u] = i < s_oldn[c] ? v.tables[(size_t)cslot[c] * v.max_pages + i] : -1;
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) dec[u] = (old[u] != nw && old[u] >= 0) ? atomicSub(&v.refcnt[old[u]], 1) : 0;
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            if (old[u] == nw) continue;
+            if (nw >= 0) ++add;
+            if (dec[u] == 1) {  // the page's last reference: it is free
+              atomicOr(&v.free_bits[old[u] >> 5], 1u << (old[u] & 31));
+              atomicMin(&s_minword, old[u] >> 5);
+              atomicAdd(&s_freed, 1);
+            }
+            if (i < new_n) v.tables[(size_t)cslot[c0 + u] * v.max_pages + i] = nw;
+          }
         }
         if (add > 0) atomicAdd(&v.refcnt[nw], add);
       }
