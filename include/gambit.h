@@ -271,6 +271,16 @@ gb_status gb_pool_status(gb_pool* pool, int* device_status, gb_stream_t stream);
 /* Reset the device status word to GB_OK (enqueued on `stream`). */
 gb_status gb_pool_clear_status(gb_pool* pool, gb_stream_t stream);
 
+/*
+ * Diagnostic of the failure path (not part of the method): enqueue one warp
+ * that waits, with the attention launch's bounded wait, for a (beam, KV head)
+ * record count that no kernel raises.  After the wait limit (2 s) it records
+ * GB_ERR_TIMEOUT in the device status and returns, leaving the context and the
+ * pool usable (clear the status to go on).  It touches no pool state but the
+ * status word; it must not overlap a decode step of the pool.
+ */
+gb_status gb_pool_wait_selftest(gb_pool* pool, gb_stream_t stream);
+
 /* Synchronise `stream` and copy the pool state into host arrays (see gb_pool_state). */
 gb_status gb_pool_read_state(gb_pool* pool, const gb_pool_state* state, gb_stream_t stream);
 

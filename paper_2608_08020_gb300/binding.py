@@ -27,7 +27,7 @@ GB_PATH_AUTO, GB_PATH_PER_BEAM, GB_PATH_GROUPED = 0, 1, 2
 # Every symbol the header declares, in header order.
 EXPORTS = ["gb_pool_workspace_bytes", "gb_pool_init", "gb_pool_destroy", "gb_pool_seed", "gb_decode_attention",
            "gb_append_kv", "gb_score_probe", "gb_push_scores", "gb_prune_branch", "gb_release", "gb_pool_status",
-           "gb_pool_clear_status", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
+           "gb_pool_clear_status", "gb_pool_wait_selftest", "gb_pool_read_state", "gb_pool_set_profile_events", "gb_pool_launch_count",
            "gb_paged_decode_noalloc", "gb_paged_decode_noalloc_status", "gb_pool_read_step_stats", "gb_pool_set_capacity", "gb_pool_last_ranked", "gb_score_mlp", "gb_fork_slots", "gb_scorer_sizes", "gb_scorer_seed",
            "gb_scorer_step", "gb_last_error"]
 GB_PROF_DECODE, GB_PROF_PROBE, GB_PROF_PRUNE, GB_PROF_GROUPED = 0, 1, 2, 3
@@ -88,6 +88,7 @@ def load(path: Path | None = None) -> ctypes.CDLL:
         "gb_release": [V, V, I, V],
         "gb_pool_status": [V, P, V],
         "gb_pool_clear_status": [V, V],
+        "gb_pool_wait_selftest": [V, V],
         "gb_pool_read_state": [V, P, V],
         "gb_pool_set_profile_events": [V, I, V, V],
         "gb_pool_launch_count": [V, P],
@@ -247,6 +248,10 @@ def gb_pool_status(pool: int, stream=None) -> int:
 
 def gb_pool_clear_status(pool: int, stream=None) -> None:
     _check(pool, load().gb_pool_clear_status(pool, stream_handle(stream)), "gb_pool_clear_status")
+
+
+def gb_pool_wait_selftest(pool: int, stream=None) -> None:
+    _check(pool, load().gb_pool_wait_selftest(pool, stream_handle(stream)), "gb_pool_wait_selftest")
 
 
 def gb_pool_read_state(pool: int, state: GbPoolState, stream=None) -> None:

@@ -551,6 +551,18 @@ static cudaError_t launch_decode_t(gb_pool* pool, int layer, const void* q, floa
   return e;
 }
 
+// One warp waits for the record count of pair 0 to reach one more than it holds; nothing
+// raises it, so the wait runs out (the same bounded wait as the attention launch's merge).
+__global__ void k_wait_selftest(PoolView v) {
+  const int have = v.pair_cnt[0];
+  if (!wait_pair_records(v, 0, have + 1, 0) && threadIdx.x == 0) set_status(v.ctl, GB_ERR_TIMEOUT);
+}
+
+cudaError_t launch_wait_selftest(gb_pool* pool, cudaStream_t s) {
+  k_wait_selftest<<<1, 32, 0, s>>>(pool->view);
+  return cudaGetLastError();
+}
+
 // Split-KV decode + combine on an explicit view (plan mode 0, W warps), for callers
 // that supply their own tables and scratch instead of a pool.
 template <int DT, int G>

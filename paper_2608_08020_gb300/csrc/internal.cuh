@@ -307,6 +307,7 @@ cudaError_t launch_decode_view(const PoolView& v, int W, int layer, const void* 
                                cudaStream_t s);
 cudaError_t rebuild_segments(gb_pool* pool, cudaStream_t s);
 cudaError_t launch_attention(gb_pool* pool, int layer, const void* q, float scale, float* out, cudaStream_t s);
+cudaError_t launch_wait_selftest(gb_pool* pool, cudaStream_t s);
 void make_kv_tensor_maps(gb_pool* pool);
 cudaError_t launch_probe(gb_pool* pool, const void* hidden, int hidden_dtype, int H, const float* w,
                          float bias, const uint8_t* mask, float* score_out, const float* scores_in,

@@ -738,6 +738,14 @@ extern "C" gb_status gb_pool_launch_count(gb_pool* pool, uint64_t* count) {
   return GB_OK;
 }
 
+extern "C" gb_status gb_pool_wait_selftest(gb_pool* pool, gb_stream_t stream) {
+  if (!pool) return GB_ERR_INVALID;
+  if (launch_wait_selftest(pool, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return check_launch(pool, "wait_selftest");
+  pool->launches += 1;
+  return check_launch(pool, "wait_selftest");
+}
+
 extern "C" gb_status gb_pool_clear_status(gb_pool* pool, gb_stream_t stream) {
   if (!pool) return GB_ERR_INVALID;
   k_clear_status<<<1, 1, 0, reinterpret_cast<cudaStream_t>(stream)>>>(pool->view);
