@@ -43,6 +43,17 @@ def test_full_size_group_sizes_match_oracle(cuda, config, hq, hkv):
                      "auto")
 
 
+# Page sizes 32 and 64 on the 512-beam tree (the per-beam CTAs following the grouped ones): the
+# grouped role's page boxes (4 and 2 pages per 128-token tile) and the per-beam role's chunks
+# inside larger pages.
+@pytest.mark.parametrize("P", [32, 64])
+def test_full_size_page_sizes_match_oracle(cuda, P):
+    import dataclasses
+
+    base = BY_INDEX[3 - 1]
+    _check_full_size(dataclasses.replace(base, name=f"{base.name}-P{P}", page_size=P), "auto")
+
+
 def _check_full_size(wl, path):
     import torch
 
