@@ -50,6 +50,7 @@ enum Ctl : int {
   kCtlBarCount = 17,   // grid-barrier arrivals of the tournament kernel (only grows)
   kCtlSegGen = 19,     // segment rebuilds so far (stamps the per-page claim words)
   kCtlSegAlloc = 20,   // words 20-21: (segments << 32 | member slots) handed out by the running rebuild
+  kCtlTailShared = 22, // 1 when a partial tail page may be shared (set by seed and forks, cleared by the planner)
   kCtlWords = 32
 };
 

@@ -196,7 +196,10 @@ __global__ void __launch_bounds__(1024) k_seed_alloc(PoolView v, int n_beams, in
     v.mean[b] = 0.f;
     v.lineage[b] = (unsigned)(lin0 + b);
   }
-  if (threadIdx.x == 0) v.ctl[kCtlNextLineage] = lin0 + n_beams;
+  if (threadIdx.x == 0) {
+    v.ctl[kCtlNextLineage] = lin0 + n_beams;
+    v.ctl[kCtlTailShared] = 1;  // the prompt's last page may be partial
+  }
 }
 
 // Copy the prompt's K/V ([layer][T][Hkv][D]) into the pages listed in slot 0's table.
@@ -236,16 +239,32 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
   __shared__ int s_tail[kMaxBeams];
   __shared__ int s_ncow, s_nact;
   __shared__ int s_tok[2];
+  __shared__ int s_ctl[8];  // free pages, steps, and the segment totals of the step record
   const int b = threadIdx.x;
+  // Every load that depends on nothing else goes out first, together.
   const bool act = b < v.max_beams && v.active[b] != 0;
   const int L = act ? v.seq_len[b] : 0;
-  if (b == 0) s_ncow = 0;
+  const int cover = (seg_cover != nullptr && b < v.max_beams) ? seg_cover[b] : 0;
+  if (b == 0) {
+    s_ncow = 0;
+    s_ctl[0] = v.ctl[kCtlFree];
+    s_ctl[1] = v.ctl[kCtlSteps];
+    s_ctl[2] = v.ctl[kCtlSegRowTok];
+    s_ctl[3] = v.ctl[kCtlSegTileTok];
+    s_ctl[4] = v.ctl[kCtlSegCount];
+    s_ctl[5] = v.ctl[kCtlSegTiles];
+    s_ctl[6] = v.ctl[kCtlSegTok];
+    s_ctl[7] = v.ctl[kCtlTailShared];
+  }
 
   // Copy-on-write decision for a still-shared partial tail page: holders
   // decide in slot order against the current refcount, so the i-th holder
-  // (1-based) copies iff i < refcnt.
+  // (1-based) copies iff i < refcnt.  Only after a seed or a fork can a partial tail page be
+  // shared; the first step after one resolves them all.
+  __syncthreads();
+  const bool tails_shared = s_ctl[7] != 0;
   int tail = -1;
-  if (act && (L % v.P) != 0) tail = v.tables[(size_t)b * v.max_pages + L / v.P];
+  if (tails_shared && act && (L % v.P) != 0) tail = v.tables[(size_t)b * v.max_pages + L / v.P];
   if (b < kMaxBeams) s_tail[b] = tail;
   __syncthreads();
   bool cow = false;
@@ -271,7 +290,7 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
   block_exclusive_scan(act ? 1 : 0, tmp, &nact);
   if (b == 0) s_nact = nact;
   const bool any_too_long = __syncthreads_or(too_long);
-  if (any_too_long || total_need > v.ctl[kCtlFree]) {
+  if (any_too_long || total_need > s_ctl[0]) {
     if (b == 0) v.ctl[kCtlCowJobs] = 0;
     if (b == 0) { set_status(v.ctl, GB_ERR_OOM); v.ctl[kCtlStepOk] = 0; }
     return;
@@ -318,7 +337,7 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
   // covered by grouped shared-prefix segments.
   for (int mode = 0; mode < 2; ++mode) {
     int start = 0;
-    if (mode == 1 && seg_cover != nullptr && act) start = seg_cover[b] * v.P;
+    if (mode == 1 && act) start = cover * v.P;
     if (start > Lnew) start = Lnew;
     const int n = act ? (Lnew - start + kChunk - 1) / kChunk : 0;
     int total;
@@ -336,21 +355,24 @@ __global__ void __launch_bounds__(1024) k_step_begin(PoolView v, int n_tokens, c
   if (b == 0) {
     // Work of this step: tokens each path reads per KV head, and the segment work of the
     // grouped path (valid until the next rebuild).
-    const int step = v.ctl[kCtlSteps];
+    const int step = s_ctl[1];
     int* e = v.stats + (size_t)(step % kStatsRing) * kStatsWords;
     e[0] = s_tok[0];
     e[1] = s_tok[1];
-    e[2] = v.grouped ? v.ctl[kCtlSegRowTok] : 0;
-    e[3] = v.grouped ? v.ctl[kCtlSegTileTok] : 0;
-    e[4] = v.grouped ? v.ctl[kCtlSegCount] : 0;
-    e[5] = v.grouped ? v.ctl[kCtlSegTiles] : 0;
+    e[2] = v.grouped ? s_ctl[2] : 0;
+    e[3] = v.grouped ? s_ctl[3] : 0;
+    e[4] = v.grouped ? s_ctl[4] : 0;
+    e[5] = v.grouped ? s_ctl[5] : 0;
     e[6] = n_tokens;
     e[7] = step;
-    e[8] = v.grouped ? v.ctl[kCtlSegTok] : 0;
+    e[8] = v.grouped ? s_ctl[6] : 0;
     e[9] = s_nact;
     v.ctl[kCtlSteps] = step + 1;
   }
-  if (b == 0) v.ctl[kCtlStepOk] = 1;
+  if (b == 0) {
+    if (tails_shared) v.ctl[kCtlTailShared] = 0;
+    v.ctl[kCtlStepOk] = 1;
+  }
 }
 
 // Write n_tokens new K/V rows per active slot for one layer at positions

@@ -54,7 +54,10 @@ __global__ void __launch_bounds__(1024) k_fork_slots(PoolView v, const int* __re
     v.active[s] = 1;
     v.lineage[s] = lin0 + tid;
   }
-  if (tid == 0) v.ctl[kCtlNextLineage] = (int)(lin0 + nchild);
+  if (tid == 0) {
+    v.ctl[kCtlNextLineage] = (int)(lin0 + nchild);
+    if (nchild > 0) v.ctl[kCtlTailShared] = 1;  // children share their parents' partial tail pages
+  }
 }
 
 }  // namespace gb

@@ -239,6 +239,8 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
     const int npar = (nchild + per - 1) / per;
     const unsigned lin0 = s_lin0;
 
+    // Children share their parents' partial tail pages until the next step's planner copies them.
+    if (blockIdx.x == 0 && tid == 0 && nchild > 0) v.ctl[kCtlTailShared] = 1;
     // Outputs (CTA 0): parent_of, pruned flags, lineage ids after the round.
     if (blockIdx.x == 0 && tid < cap) {
       const int k = childof[tid];
