@@ -86,6 +86,28 @@ def test_noalloc_matches_oracle_on_caller_tables_two_calls(cuda, dtype, G, P):
         _check_rows(c, d["out"].cpu().numpy(), f"{dtype} G={G} P={P} call {call}")
 
 
+@pytest.mark.parametrize("dtype,G,P", [("f32", 4, 16), ("bf16", 4, 16), ("bf16", 8, 64)])
+def test_noalloc_is_invariant_to_physical_page_placement(cuda, dtype, G, P):
+    """The same logical K/V stored in other physical pages (the pool permuted, the tables
+    renumbered to follow) gives bit-identical outputs: only the table decides which page holds
+    which tokens."""
+    from paper_2608_08020_gb300 import binding as B
+    c = _case(dtype, G, P, seed=7 * G + P)
+    d = _device(c, cuda)
+    assert _call(B, c, d) == B.GB_OK
+    first = d["out"].cpu().numpy()
+    perm = np.random.default_rng(11).permutation(c["num_pages"])   # new page of old page i: perm[i]
+    c2 = dict(c)
+    kv2 = np.empty_like(c["kv"])
+    kv2[perm] = c["kv"]
+    c2["kv"] = kv2
+    c2["tables"] = perm[c["tables"]].astype(np.int32)
+    d2 = _device(c2, cuda)
+    assert _call(B, c2, d2) == B.GB_OK
+    second = d2["out"].cpu().numpy()
+    assert np.array_equal(first, second), np.abs(first - second).max()
+
+
 def test_noalloc_row_longer_than_its_table_is_refused_and_reported(cuda):
     from paper_2608_08020_gb300 import binding as B
     c = _case("bf16", 4, 16, seed=7)
