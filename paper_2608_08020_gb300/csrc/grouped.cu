@@ -122,6 +122,15 @@ __device__ __forceinline__ void tma_page(uint32_t dst, const CUtensorMap* tm, in
       "l"(tm), "r"(0), "r"(0), "r"(0), "r"(kv), "r"(w), "r"(bar)
       : "memory");
 }
+// The same with an L2 eviction policy (a page no other query tile of its segment reads again).
+__device__ __forceinline__ void tma_page_hint(uint32_t dst, const CUtensorMap* tm, int kv, int w, uint32_t bar,
+                                              uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7], %8;" ::"r"(dst),
+      "l"(tm), "r"(0), "r"(0), "r"(0), "r"(kv), "r"(w), "r"(bar), "l"(pol)
+      : "memory");
+}
 
 // Everything a role needs to know about one unit of work.
 struct Unit {
@@ -206,6 +215,7 @@ __device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMa
     if (lane == 0) asm volatile("prefetch.tensormap [%0];" ::"l"(tm_p) : "memory");
     const int ppt = kTok / v.P;                     // pages per tile (2 to 16)
     const uint32_t page_bytes = (uint32_t)v.P * 256;  // K (or V) of one page of one head
+    const uint64_t pol_ef = policy_evict_first();
     uint32_t n = 0;  // tiles issued
     int uidx = 0;    // units started
     bool ok = true;
@@ -286,7 +296,14 @@ __device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMa
         __syncwarp();
         // Lane c issues page c: a TMA instruction holds its thread for a while, so the
         // lanes' copies go out in parallel.
-        if (lane < ppt) tma_page(sbase + kKRing + st * kHalfStage + lane * page_bytes, tm_p, 0, w, bar);
+        if (lane < ppt) {
+          // The segment's only query tile reads its pages once: evict them first, before data
+          // that is read again (the queries, the records, other tiles' pages).
+          if (x.g * G <= kRows)
+            tma_page_hint(sbase + kKRing + st * kHalfStage + lane * page_bytes, tm_p, 0, w, bar, pol_ef);
+          else
+            tma_page(sbase + kKRing + st * kHalfStage + lane * page_bytes, tm_p, 0, w, bar);
+        }
         if (j == 0) {
           // Query rows of the unit (after its first tile's copies are under way): row r =
           // (member, query head of this KV head); zero rows past the members.  The single
@@ -330,6 +347,7 @@ __device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMa
     // ------------------------------------------------------------------ V producer
     const int ppt = kTok / v.P;
     const uint32_t page_bytes = (uint32_t)v.P * 256;
+    const uint64_t pol_ef = policy_evict_first();
     uint32_t n = 0;  // tiles issued
     bool ok = true;
     for (int uidx = 0; ok; ++uidx) {
@@ -368,7 +386,14 @@ __device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMa
         const uint32_t bar = ctl + kBarVFull + 8 * st;
         if (lane == 0) mbar_arrive_expect_tx(bar, kHalfStage);
         __syncwarp();
-        if (lane < ppt) tma_page(sbase + kVRing + st * kHalfStage + lane * page_bytes, tm_p, 1, w, bar);
+        if (lane < ppt) {
+          // The segment's only query tile reads its pages once: evict them first, before data
+          // that is read again (the queries, the records, other tiles' pages).
+          if (x.g * G <= kRows)
+            tma_page_hint(sbase + kVRing + st * kHalfStage + lane * page_bytes, tm_p, 1, w, bar, pol_ef);
+          else
+            tma_page(sbase + kVRing + st * kHalfStage + lane * page_bytes, tm_p, 1, w, bar);
+        }
       }
     }
     if (lane == 0 && *abort_flag) {
