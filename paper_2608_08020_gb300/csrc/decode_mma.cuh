@@ -175,7 +175,10 @@ __device__ __forceinline__ void decode_mma_body(const PoolView& v, const CUtenso
     it.h = rr / it.n;
     it.i = rr % it.n;
   }
-  const uint64_t pol = policy_evict_first();
+  // L2 policy of the K/V chunks: evict first, as each is read once, unless this is the
+  // per-beam path over a tree with shared pages, where siblings read the same pages again.
+  const bool reread = mode == 0 && v.grouped && v.ctl[kCtlSegCount] > 0;
+  const uint64_t pol = reread ? policy_evict_normal() : policy_evict_first();
   int pw_b = -1, pw_i0 = 0, pw_lane = 0;
   auto load_page = [&](const ChunkIter& qi) -> int {
     if (qi.b != pw_b || qi.i < pw_i0 || qi.i >= pw_i0 + 32) {
