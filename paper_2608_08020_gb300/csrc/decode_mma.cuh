@@ -365,18 +365,19 @@ __device__ __forceinline__ void decode_mma_body(const PoolView& v, const CUtenso
       if (2 * c < G) {
         float* o0 = rec + (2 * c) * D + r;
         float* o1 = o0 + D;
+        const uint64_t rpol = policy_evict_last();  // the merge reads the record back from L2
 #pragma unroll
         for (int mt = 0; mt < 8; ++mt) {
-          o0[16 * mt] = o[mt][0];
-          o1[16 * mt] = o[mt][1];
-          o0[16 * mt + 8] = o[mt][2];
-          o1[16 * mt + 8] = o[mt][3];
+          st_hint(o0 + 16 * mt, o[mt][0], rpol);
+          st_hint(o1 + 16 * mt, o[mt][1], rpol);
+          st_hint(o0 + 16 * mt + 8, o[mt][2], rpol);
+          st_hint(o1 + 16 * mt + 8, o[mt][3], rpol);
         }
         if (r == 0) {
-          rec[G * D + 2 * c] = m0;
-          rec[G * D + 2 * c + 1] = m1;
-          rec[G * D + G + 2 * c] = l0;
-          rec[G * D + G + 2 * c + 1] = l1;
+          st_hint(rec + G * D + 2 * c, m0, rpol);
+          st_hint(rec + G * D + 2 * c + 1, m1, rpol);
+          st_hint(rec + G * D + G + 2 * c, l0, rpol);
+          st_hint(rec + G * D + G + 2 * c + 1, l1, rpol);
         }
       }
       record_arrive(v, it.b * v.Hkv + it.h, lane);

@@ -649,6 +649,7 @@ __device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMa
       const int b = bk / kMaxSegDepth;
       const bool has = m < x.g && r_idx < kMaxSegRecords;
       float* rec = v.grec + (((size_t)b * kMaxSegRecords + r_idx) * v.Hkv + x.h) * v.record_floats;
+      const uint64_t rpol = policy_evict_last();  // the merge reads the record back from L2
       // Group k writes columns [64k, 64k + 64) of the output.
 #pragma unroll 1
       for (int c0 = 0; c0 < 64; c0 += 32) {  // warp-collective loads: every lane takes part
@@ -657,12 +658,12 @@ __device__ __forceinline__ void grouped_body(const PoolView& v, const CUtensorMa
         if (has) {
 #pragma unroll
           for (int i = 0; i < 32; i += 4)
-            *reinterpret_cast<float4*>(rec + gg * 128 + grp * 64 + c0 + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
+            st_hint4(rec + gg * 128 + grp * 64 + c0 + i, make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]), rpol);
         }
       }
       if (has && grp == 0) {
-        rec[G * 128 + gg] = m_ref;
-        rec[G * 128 + G + gg] = l_all;
+        st_hint(rec + G * 128 + gg, m_ref, rpol);
+        st_hint(rec + G * 128 + G + gg, l_all, rpol);
       }
       tc_fence_before();
       __syncwarp();
