@@ -132,6 +132,12 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
 
   const int tid = threadIdx.x;
   const int cap = v.max_beams;
+  // The slot's state for the ranking, loaded first and together.
+  const bool in = a.prune && tid < cap;
+  const int act_w = in ? v.active[tid] : 0;
+  const int gen_w = in ? v.gen[tid] : 0;
+  const float mean_w = in ? v.mean[tid] : 0.f;
+  const int elig_w = (in && a.elig != nullptr) ? a.elig[tid] : 1;
   if (tid == 0) {
     s_fail = 0;
     s_nchild = 0;
@@ -153,8 +159,8 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
 
   // ---- 1. tournament ---------------------------------------------------------------------
   if (a.prune) {
-    const bool act = tid < cap && v.active[tid] != 0;
-    const bool elig = act && v.gen[tid] >= a.warmup && (a.elig == nullptr || a.elig[tid] != 0);
+    const bool act = act_w != 0;
+    const bool elig = act && gen_w >= a.warmup && elig_w != 0;
     s_act[tid] = act;
     s_elig[tid] = elig;
     s_pruned[tid] = 0;
@@ -163,7 +169,7 @@ __global__ void __launch_bounds__(kTourThreads, 1) k_tournament(PoolView v, Tour
     const int pos = block_exclusive_scan(act ? 1 : 0, tmp, &N);
     s_keys[tid] = ~0ull;
     __syncthreads();
-    if (act) s_keys[pos] = ((unsigned long long)rank_key(v.mean[tid]) << 32) | (unsigned)tid;
+    if (act) s_keys[pos] = ((unsigned long long)rank_key(mean_w) << 32) | (unsigned)tid;
     __syncthreads();
     // Rank (ascending keys; the slot in the low word makes them distinct): each warp sorts its
     // 32 keys in registers (bitonic, by shuffles), then a key's rank is its position in its
