@@ -6,15 +6,16 @@
 // number w + b * Hkv + h), and, on the grouped path, nseg records of the beam's shared-prefix
 // segments.  A per-beam warp counts each record it writes in pair_cnt[b * Hkv + h] (release:
 // fence, then the add); a grouped CTA counts itself in ctl[kCtlGrpDone] once all of its
-// records are written.  After its own work, every warp of the grid takes the pairs
-// p = cta + nctas * (warp + k * warps per CTA), waits (bounded) until pair_cnt[p] == npb
-// and, when nseg > 0, every grouped CTA has finished, then merges the R records into
-// out[b][h * G + g][:]: running max M of the records' m, acc = sum o * 2^(m - M),
-// L = sum l * 2^(m - M), out = acc / L.
+// records are written.  After their own work, the merging CTAs (the launch's caller names
+// them: cta of nctas) take the pairs p = cta + nctas * (warp + k * warps per CTA); a warp waits
+// (bounded) until pair_cnt[p] == npb and, when nseg > 0, every grouped CTA has finished, then
+// merges the R records into out[b][h * G + g][:]: running max M of the records' m,
+// acc = sum o * 2^(m - M), L = sum l * 2^(m - M), out = acc / L.
 //
-// All CTAs of these kernels are resident together (one per SM, grid = SM count), so the
-// waits end; each is bounded and gives up as soon as the pool's status word is set.  The
-// counters are zeroed by k_append, the launch that precedes every attention launch.
+// The waits end because every CTA they wait on gets an SM: the callers only let CTAs merge
+// that are resident together with the ones they wait on, or that wait only on CTAs which never
+// wait (k_attention).  Each wait is bounded and gives up as soon as the pool's status word is
+// set.  The counters are zeroed by k_append, the launch that precedes every attention launch.
 #pragma once
 #include <cuda_runtime.h>
 #include <math.h>
