@@ -489,7 +489,6 @@ def run_ours(args) -> None:
     K = args.steps if args.steps > 0 else default_steps(wl, W, Kp, with_e2e, step_input_bytes)
     lay = step_layout(wl, K, Kp, W, with_e2e)
     delta = wl.interval
-    capacity = capacity_search(wl, dev) if (wl.pool_bytes is not None and rank == 0 and not args.no_capacity) else None
 
     # Every phase ends at or before the workload's context, so the pool needs tables of that length.
     fixed_pool = wl.pool_bytes is not None
@@ -857,6 +856,10 @@ def run_ours(args) -> None:
 
     value = job_value(world, C, K, elapsed_ms)
     ms_per_step = elapsed_ms / K
+
+    # The capacity search builds and frees about a dozen one-layer pools; it runs after every timed
+    # phase so that none of them runs in the state it leaves (host and device allocations).
+    capacity = capacity_search(wl, dev) if (wl.pool_bytes is not None and rank == 0 and not args.no_capacity) else None
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
