@@ -10,10 +10,10 @@ a fork, or at the end - is scored once and checked at every recorded position). 
 step pool's pages are compared bit for bit with ``oracle.pool.PoolOracle`` replaying
 the same seed, steps, forks and releases.
 
-Tolerance: |device - oracle| <= 1.5e-2 on the score.  The device rounds to bf16 the
-operands of every product (LayerNorm outputs, q/k/v, attention and SwiGLU outputs);
-replaying exactly those roundings in numpy against the fp64 oracle gives at most
-4.1e-3 over 18 seeded shapes of 30 positions, and fp32 accumulation adds far less.
+Tolerance: |device - oracle| <= 8e-3 on the score, twice the bf16 bound: the device
+rounds to bf16 the operands of every product (LayerNorm outputs, q/k/v, attention and
+SwiGLU outputs); replaying exactly those roundings in numpy against the fp64 oracle gives
+at most 4.1e-3 over 18 seeded shapes of 30 positions, and fp32 accumulation adds far less.
 """
 import numpy as np
 import pytest
@@ -25,7 +25,7 @@ from workload.scorer_weights import _bf16, seqscorer_weights
 
 pytestmark = pytest.mark.gpu
 
-ATOL = 1.5e-2
+ATOL = 8e-3
 
 
 def _oracle_weights(w: dict) -> SeqScorerWeights:
