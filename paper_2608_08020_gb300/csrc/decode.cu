@@ -420,7 +420,7 @@ __global__ void __launch_bounds__(kMmaWarps * 32, 1)
   pdl_wait();
   pdl_launch_dependents();
   decode_mma_body<G>(v, &tm, &tmh, layer, q, qscale, mode, (int)blockIdx.x, (int)gridDim.x);
-  combine_pairs<G>(v, mode, (int)gridDim.x * kMmaWarps, 0, (int)blockIdx.x, (int)gridDim.x, out);
+  combine_pairs<G>(v, mode, (int)gridDim.x * kMmaWarps, 0, false, (int)blockIdx.x, (int)gridDim.x, out);
 }
 
 // Merge the partial records of each (beam, kv head) into out[b][h*G+g][:]: the split-KV

@@ -725,8 +725,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   } else {
     decode_mma_body<G>(v, &tmd, &tmdh, layer, q, qscale, 1, c - pb0, nd);
   }
-  if (split) combine_pairs<G>(v, 1, nd * kMmaWarps, ng, c, S, out);
-  else combine_pairs<G>(v, 1, nd * kMmaWarps, ng, c - S, S, out);
+  // A large step's per-beam CTAs start as grouped CTAs leave, so they take the pairs as they
+  // finish; a small step's CTAs all start together and split the pairs evenly.
+  if (split) combine_pairs<G>(v, 1, nd * kMmaWarps, ng, false, c, S, out);
+  else combine_pairs<G>(v, 1, nd * kMmaWarps, ng, true, c - S, S, out);
 }
 
 }  // namespace

@@ -51,6 +51,7 @@ enum Ctl : int {
   kCtlSegGen = 19,     // segment rebuilds so far (stamps the per-page claim words)
   kCtlSegAlloc = 20,   // words 20-21: (segments << 32 | member slots) handed out by the running rebuild
   kCtlTailShared = 22, // 1 when a partial tail page may be shared (set by seed and forks, cleared by the planner)
+  kCtlPairNext = 23,   // next (beam, KV head) pair to merge in the attention launch (zeroed by k_append)
   kCtlWords = 32
 };
 

@@ -387,6 +387,7 @@ __global__ void k_append(PoolView v, int layer, int n_tokens, const char* kin, c
     if (threadIdx.x == 0) {
       v.ctl[kCtlGrpNext] = 0;
       v.ctl[kCtlGrpDone] = 0;
+      v.ctl[kCtlPairNext] = 0;
     }
   }
   if (v.ctl[kCtlStepOk] == 0) return;
